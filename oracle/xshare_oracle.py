@@ -1,0 +1,466 @@
+"""Plain CPU oracle for one XShare MoE layer forward (arxiv 2602.07265).
+
+TEST INFRASTRUCTURE ONLY.  This module is the slow, obviously-correct
+restatement of the method that the CUDA library is checked against.  Only the
+tests, ``__graft_entry__.smoke()`` and the CPU-baseline leg of ``bench.py`` may
+import it.  It shares no code with the CUDA path and imports nothing from the
+product package.
+
+What it computes, in the paper's order and notation:
+
+* Router logits  h = W_g x                                 (Sec. 2.2)
+* Dense softmax gating scores g_ij over all N experts      (Sec. 2.2, Sec. 3.1;
+  dense reading, see ``softmax_scores``)
+* Warm-up set S_0 = union of per-token top-k0              (Sec. 3.4, Algorithm 2)
+* Column scores scores[j] = sum_i g_ij                      (Algorithm 1, Eq. 2)
+* Budgeted selection:
+    - BATCH  : Algorithm 2 with Algorithm 1 in fixed-budget form
+    - HIER   : Algorithm 4 calling Algorithm 3 per request, Eq. 3-4
+    - GROUP  : Algorithm 6 calling Algorithm 5, Eq. 5
+    - TOPK   : S = E, i.e. plain top-k routing (Sec. 2.2)
+* Refinement: each token routed to Top k(G_i, S) with renormalised weights
+                                                            (Sec. 2.2, Algorithms 2/4/6)
+* Permutation of (token, slot) pairs by expert (counting sort, stable)
+* Expert FFN E_i(x) = W_down (silu(W_gate x) * (W_up x)) over the pairs, and the
+  weighted combine y = sum_i g_i(x) E_i(x) of the routed part  (Sec. 2.1)
+
+Precision.  Selection is decided on fp32 scores (the precision the kernels
+decide in): softmax is evaluated in fp64 and rounded to fp32 once, column sums
+use the canonical fp32 order defined in ``canonical_column_sum``, the
+renormalised weights are fp32.  Router logits and the expert FFN are fp64.
+
+Readings of the paper where it is silent or ambiguous are stated at each
+function; every one of them is listed in the design notes of the repository.
+"""
+
+from __future__ import annotations
+
+import math
+from typing import Dict, List, Optional, Sequence, Set, Tuple
+
+import numpy as np
+
+MODE_TOPK = 0
+MODE_BATCH = 1
+MODE_GROUP = 2
+MODE_HIER = 3
+
+MODE_NAMES = {MODE_TOPK: "topk", MODE_BATCH: "batch", MODE_GROUP: "group", MODE_HIER: "hier"}
+
+# Width of one chunk of the canonical column sum (one warp of 32 lanes).
+CHUNK = 32
+
+
+# --------------------------------------------------------------------------
+# Number formats
+# --------------------------------------------------------------------------
+
+def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
+    """Widen raw bf16 bit patterns (uint16) to float64 exactly.
+
+    A bf16 value is the upper 16 bits of an IEEE binary32 value, so shifting
+    the pattern left by 16 gives the fp32 number, which fp64 holds exactly.
+    """
+    b = np.asarray(bits, dtype=np.uint16)
+    return (b.astype(np.uint32) << np.uint32(16)).view(np.float32).astype(np.float64)
+
+
+# --------------------------------------------------------------------------
+# Sec. 2.2: router logits and gating scores
+# --------------------------------------------------------------------------
+
+def router_logits(x_bits: np.ndarray, W_g: np.ndarray) -> np.ndarray:
+    """h(x) = W_g x for every token (Sec. 2.2), in fp64.
+
+    x_bits: [B, d] uint16 bf16 patterns; W_g: [N, d] float32.  Returns [B, N]
+    float64.  The bf16 inputs and fp32 weights are widened exactly; the dot
+    products use fp64 arithmetic.
+    """
+    x = bf16_bits_to_f64(x_bits)
+    W = np.asarray(W_g, dtype=np.float32).astype(np.float64)
+    return x @ W.T
+
+
+def softmax_scores(h: np.ndarray) -> np.ndarray:
+    """Gating scores g_ij = exp(h_ij) / sum_j' exp(h_ij') over ALL N experts.
+
+    Reading of Sec. 2.2 / Sec. 3.1: the scores G_i that the selection step sums
+    are the dense softmax over the full expert set, not the top-k-masked ones;
+    only dense scores make "top-k within S" (the refinement step) meaningful.
+    Evaluated in fp64 (row maximum subtracted first), then rounded once to
+    fp32, the precision in which every selection decision is taken.
+    """
+    h = np.asarray(h, dtype=np.float64)
+    z = h - h.max(axis=1, keepdims=True)
+    e = np.exp(z)
+    return (e / e.sum(axis=1, keepdims=True)).astype(np.float32)
+
+
+# --------------------------------------------------------------------------
+# Total order used by every top-k / argmax of the method
+# --------------------------------------------------------------------------
+
+def ranked(values: np.ndarray, candidates: Sequence[int]) -> List[int]:
+    """Candidates sorted best-first: larger value first, ties to the lower index.
+
+    The paper does not say how ties break; the lower expert index wins
+    everywhere.  Values are fp32 and compared exactly.
+    """
+    return sorted(candidates, key=lambda j: (-float(values[j]), j))
+
+
+def top(values: np.ndarray, count: int, candidates: Sequence[int]) -> List[int]:
+    """Top `count` of `candidates` under the total order (fewer if not enough)."""
+    if count <= 0:
+        return []
+    return ranked(values, candidates)[:count]
+
+
+# --------------------------------------------------------------------------
+# Algorithm 1 / Eq. 2: column scores
+# --------------------------------------------------------------------------
+
+def canonical_column_sum(p: np.ndarray, rows: Sequence[int]) -> np.ndarray:
+    """scores[j] = sum over the given rows i of g_ij, in the canonical fp32 order.
+
+    The paper does not fix a summation order.  Selection compares these sums,
+    so the order is fixed here and the kernels follow the same one:
+
+    * the rows are taken in the given order and split into chunks of 32,
+      the last chunk padded with zeros;
+    * inside a chunk of values v[0..31] a halving tree is applied:
+      for o = 16, 8, 4, 2, 1: v[l] <- v[l] + v[l + o] for every l < o;
+      the chunk's sum is v[0];
+    * chunk sums are added left to right to an accumulator that starts at 0.
+
+    Every addition is one fp32 addition rounded to nearest.  Returns [N] float32.
+    """
+    p = np.asarray(p, dtype=np.float32)
+    N = p.shape[1]
+    rows = list(rows)
+    acc = np.zeros(N, dtype=np.float32)
+    for c0 in range(0, len(rows), CHUNK):
+        chunk_rows = rows[c0:c0 + CHUNK]
+        v = np.zeros((CHUNK, N), dtype=np.float32)
+        v[:len(chunk_rows)] = p[chunk_rows]
+        o = CHUNK // 2
+        while o >= 1:
+            v[:o] = v[:o] + v[o:2 * o]
+            o //= 2
+        acc = acc + v[0]
+    return acc
+
+
+# --------------------------------------------------------------------------
+# Warm-up initialisation (Sec. 3.4)
+# --------------------------------------------------------------------------
+
+def warmup_set(p: np.ndarray, k0: int, tokens: Sequence[int]) -> Set[int]:
+    """S_0 = union over the given tokens of Top k0(G_i, E) (Algorithms 2, 3, 6)."""
+    N = p.shape[1]
+    S0: Set[int] = set()
+    for i in tokens:
+        S0.update(top(p[i], k0, range(N)))
+    return S0
+
+
+# --------------------------------------------------------------------------
+# Selection algorithms
+# --------------------------------------------------------------------------
+
+def greedy_select_budget(scores: np.ndarray, m: int, S0: Set[int]) -> Set[int]:
+    """Algorithm 1 in the fixed-budget form used in practice (Sec. 3.4).
+
+    Starting from S_0, repeatedly add argmax_{e in E \\ S} scores[e], m times
+    (or until E is exhausted).  Reading: the budget m counts experts added
+    beyond S_0, as Algorithm 3 writes explicitly (S_0 union Top m_r).
+    By Proposition 1 the marginal gain of e is scores[e] whatever S is, so the
+    argmax is taken over the precomputed column scores.
+    """
+    N = scores.shape[0]
+    S = set(S0)
+    for _ in range(m):
+        rest = [e for e in range(N) if e not in S]
+        if not rest:
+            break
+        S.add(ranked(scores, rest)[0])
+    return S
+
+
+def select_batch(p: np.ndarray, m: int, k0: int) -> Tuple[Set[int], Set[int]]:
+    """Algorithm 2: warm-up S_0, then GreedySelect with budget m.  Returns (S, S_0)."""
+    B = p.shape[0]
+    S0 = warmup_set(p, k0, range(B))
+    scores = canonical_column_sum(p, range(B))
+    return greedy_select_budget(scores, m, S0), S0
+
+
+def per_request_select(p: np.ndarray, tokens: Sequence[int], m_r: int, k0: int) -> Set[int]:
+    """Algorithm 3 for one request r with tokens T_r.
+
+    S_0 = union of Top k0 over T_r; scores[j] = sum over T_r of g_xj (Eq. 3);
+    S_r = S_0 union Top m_r(scores, E \\ S_0).
+    """
+    N = p.shape[1]
+    S0 = warmup_set(p, k0, tokens)
+    scores = canonical_column_sum(p, tokens)
+    rest = [e for e in range(N) if e not in S0]
+    return S0 | set(top(scores, m_r, rest))
+
+
+def select_hier(p: np.ndarray, m: int, m_r: int, k0: int,
+                tokens_per_request: int) -> Tuple[Set[int], Set[int]]:
+    """Algorithm 4: union of per-request selections, then GreedySelect(m).
+
+    Requests are contiguous runs of `tokens_per_request` = 1 + L_s tokens
+    (Sec. 4.1).  Returns (S_batch, union of the S_r before the batch step).
+    """
+    B = p.shape[0]
+    T = tokens_per_request
+    S_b: Set[int] = set()
+    for r in range(B // T):
+        S_b |= per_request_select(p, range(r * T, (r + 1) * T), m_r, k0)
+    scores = canonical_column_sum(p, range(B))
+    return greedy_select_budget(scores, m, S_b), S_b
+
+
+def group_of(e: int, N: int, G: int) -> int:
+    """Index of the group E_g holding expert e: G contiguous ranges of N/G."""
+    return e // (N // G)
+
+
+def gpu_aware_greedy(scores: np.ndarray, G: int, m_g: int, S0: Set[int]) -> Set[int]:
+    """Algorithm 5 taken literally.
+
+    S = S_0; while |S| < m_g * G: for g = 1..G: add the argmax of the marginal
+    gain over E_g \\ S (the column score, by Proposition 1).
+    Readings: a round always runs over all G groups, so |S| may end above
+    m_g * G by up to G - 1; a group with nothing left is skipped; when every
+    group is exhausted the loop stops (the pseudocode would not terminate).
+    """
+    N = scores.shape[0]
+    size = N // G
+    S = set(S0)
+    while len(S) < m_g * G:
+        added = False
+        for g in range(G):
+            rest = [e for e in range(g * size, (g + 1) * size) if e not in S]
+            if not rest:
+                continue
+            S.add(ranked(scores, rest)[0])
+            added = True
+        if not added:
+            break
+    return S
+
+
+def select_group(p: np.ndarray, G: int, m_g: int, k0: int) -> Tuple[Set[int], Set[int]]:
+    """Algorithm 6: warm-up S_0 over the batch, then Algorithm 5.  Returns (S, S_0)."""
+    B = p.shape[0]
+    S0 = warmup_set(p, k0, range(B))
+    scores = canonical_column_sum(p, range(B))
+    return gpu_aware_greedy(scores, G, m_g, S0), S0
+
+
+# --------------------------------------------------------------------------
+# Refinement (Sec. 3.4) with renormalised weights (Sec. 2.2)
+# --------------------------------------------------------------------------
+
+def refine(p: np.ndarray, S: Set[int], k: int) -> Tuple[np.ndarray, np.ndarray]:
+    """Route every token to Top k(G_i, S) and renormalise.
+
+    k' = min(k, |S|) experts per token, listed best-first; slots k'..k-1 hold
+    id -1 and weight 0 (reading for |S| < k).  The weight of a routed expert
+    follows Sec. 2.2 restricted to the routed set T':
+        g_bar = exp(h_e) / sum_{j in T'} exp(h_j) = g_e / sum_{j in T'} g_j,
+    with the denominator D the fp32 sum of the k' scores in slot order and one
+    fp32 division.  If D is 0 (every score underflowed) each weight is 1/k'.
+    Returns ids [B, k] int32 and weights [B, k] float32.
+    """
+    p = np.asarray(p, dtype=np.float32)
+    B = p.shape[0]
+    kp = min(k, len(S))
+    cands = sorted(S)
+    ids = np.full((B, k), -1, dtype=np.int32)
+    w = np.zeros((B, k), dtype=np.float32)
+    for i in range(B):
+        chosen = top(p[i], kp, cands)
+        D = np.float32(0.0)
+        for e in chosen:
+            D = np.float32(D + p[i, e])
+        for s, e in enumerate(chosen):
+            ids[i, s] = e
+            if D > 0:
+                w[i, s] = np.float32(p[i, e] / D)
+            else:
+                w[i, s] = np.float32(np.float32(1.0) / np.float32(kp))
+    return ids, w
+
+
+# --------------------------------------------------------------------------
+# Token permutation
+# --------------------------------------------------------------------------
+
+def permute(ids: np.ndarray, N: int) -> Dict[str, np.ndarray]:
+    """Counting sort of the (token, slot) pairs by expert.
+
+    Pair id = t * k + slot.  counts[e] = pairs routed to e; offsets = exclusive
+    prefix of counts (length N + 1); perm lists pair ids grouped by expert in
+    ascending expert order and, inside an expert, in ascending (token, slot)
+    order; used = experts with at least one pair, ascending.
+    """
+    B, k = ids.shape
+    counts = np.zeros(N, dtype=np.int32)
+    for t in range(B):
+        for s in range(k):
+            e = int(ids[t, s])
+            if e >= 0:
+                counts[e] += 1
+    offsets = np.zeros(N + 1, dtype=np.int32)
+    for e in range(N):
+        offsets[e + 1] = offsets[e] + counts[e]
+    fill = offsets[:N].copy()
+    perm = np.zeros(int(offsets[N]), dtype=np.int32)
+    for t in range(B):
+        for s in range(k):
+            e = int(ids[t, s])
+            if e >= 0:
+                perm[fill[e]] = t * k + s
+                fill[e] += 1
+    used = np.array([e for e in range(N) if counts[e] > 0], dtype=np.int32)
+    return {"counts": counts, "offsets": offsets, "perm": perm, "used": used}
+
+
+# --------------------------------------------------------------------------
+# Full routing step
+# --------------------------------------------------------------------------
+
+def route(p: np.ndarray, k: int, budget: int, mode: int, k0: int = 0, m_r: int = 0,
+          tokens_per_request: int = 1, n_groups: int = 1, m_g: int = 0) -> Dict[str, object]:
+    """Batch-aware selection and refinement on fp32 gating scores p [B, N].
+
+    mode TOPK : S = E (standard top-k routing, the paper's baseline)
+    mode BATCH: Algorithm 2 with budget m = `budget`, warm-up k0
+    mode HIER : Algorithm 4 with batch budget m = `budget`, per-request m_r, k0
+    mode GROUP: Algorithm 6 with G = n_groups contiguous groups, per-group m_g, k0
+    Returns the selected mask, the routing, the permutation and the statistics
+    |S|, |U|, |union of plain top-k| and max_g |S intersect E_g|.
+    """
+    p = np.asarray(p, dtype=np.float32)
+    B, N = p.shape
+    if mode == MODE_TOPK:
+        S = set(range(N))
+    elif mode == MODE_BATCH:
+        S, _ = select_batch(p, budget, k0)
+    elif mode == MODE_HIER:
+        S, _ = select_hier(p, budget, m_r, k0, tokens_per_request)
+    elif mode == MODE_GROUP:
+        S, _ = select_group(p, n_groups, m_g, k0)
+    else:
+        raise ValueError(f"unknown mode {mode}")
+    ids, w = refine(p, S, k)
+    perm = permute(ids, N)
+    union = warmup_set(p, k, range(B))
+    G = n_groups if n_groups >= 1 else 1
+    loads = [0] * G
+    for e in S:
+        loads[group_of(e, N, G)] += 1
+    mask = np.zeros(N, dtype=np.uint8)
+    for e in S:
+        mask[e] = 1
+    return {
+        "mask": mask, "ids": ids, "w": w, **perm,
+        "n_selected": len(S), "n_used": int(len(perm["used"])),
+        "union_topk": len(union), "max_group_load": max(loads),
+    }
+
+
+# --------------------------------------------------------------------------
+# Sec. 2.1: expert FFN and weighted combine
+# --------------------------------------------------------------------------
+
+def silu(z: np.ndarray) -> np.ndarray:
+    """silu(z) = z / (1 + exp(-z)), fp64."""
+    return z / (1.0 + np.exp(-z))
+
+
+def expert_ffn(x_rows: np.ndarray, Wgate_e: np.ndarray, Wup_e: np.ndarray,
+               Wdown_e: np.ndarray) -> np.ndarray:
+    """SwiGLU expert E_e(x) = W_down (silu(W_gate x) * (W_up x)) for a stack of x rows.
+
+    x_rows [n, d] float64; Wgate_e, Wup_e: [F, d] uint16 bf16 patterns;
+    Wdown_e: [d, F] uint16.  fp64 throughout.  Returns [n, d] float64.
+    """
+    g = x_rows @ bf16_bits_to_f64(Wgate_e).T
+    u = x_rows @ bf16_bits_to_f64(Wup_e).T
+    a = silu(g) * u
+    return a @ bf16_bits_to_f64(Wdown_e).T
+
+
+def combine(ids: np.ndarray, w: np.ndarray, expert_out: Dict[Tuple[int, int], np.ndarray],
+            tokens: Sequence[int], d: int) -> np.ndarray:
+    """Routed part of the layer output, y_t = sum over slots of w_ts * E_{ids_ts}(x_t).
+
+    `expert_out[(t, s)]` is the expert output for pair (t, s).  Slots with id -1
+    contribute nothing.  fp64, weights widened from fp32.  Returns [len(tokens), d].
+    """
+    y = np.zeros((len(tokens), d), dtype=np.float64)
+    for r, t in enumerate(tokens):
+        for s in range(ids.shape[1]):
+            if ids[t, s] >= 0:
+                y[r] += float(w[t, s]) * expert_out[(t, s)]
+    return y
+
+
+def moe_ffn_combine(x_bits: np.ndarray, ids: np.ndarray, w: np.ndarray,
+                    get_expert, tokens: Optional[Sequence[int]] = None) -> np.ndarray:
+    """Expert FFN over the routed pairs of `tokens` and the weighted combine.
+
+    get_expert(e) -> (Wgate_e [F, d], Wup_e [F, d], Wdown_e [d, F]) as uint16
+    bf16 patterns; only experts some listed token is routed to are requested,
+    one at a time.  Returns y [len(tokens), d] float64 (all tokens by default).
+    """
+    B, k = ids.shape
+    d = x_bits.shape[1]
+    if tokens is None:
+        tokens = list(range(B))
+    x = bf16_bits_to_f64(x_bits)
+    pairs_of: Dict[int, List[Tuple[int, int]]] = {}
+    for t in tokens:
+        for s in range(k):
+            e = int(ids[t, s])
+            if e >= 0:
+                pairs_of.setdefault(e, []).append((t, s))
+    out: Dict[Tuple[int, int], np.ndarray] = {}
+    for e in sorted(pairs_of):
+        Wg, Wu, Wd = get_expert(e)
+        pairs = pairs_of[e]
+        o = expert_ffn(x[[t for t, _ in pairs]], Wg, Wu, Wd)
+        for r, ts in enumerate(pairs):
+            out[ts] = o[r]
+    return combine(ids, w, out, tokens, d)
+
+
+def moe_forward(x_bits: np.ndarray, W_g: np.ndarray, get_expert, k: int, budget: int,
+                mode: int, tokens: Optional[Sequence[int]] = None, **params) -> Dict[str, object]:
+    """One MoE layer forward: router, dense softmax, selection, refinement,
+    permutation, expert FFN over the routed pairs and weighted combine.
+
+    Returns the routing dictionary of `route` plus "h" (fp64 logits), "p" (fp32
+    scores) and "y" (fp64 routed output for `tokens`, all by default).
+    """
+    h = router_logits(x_bits, W_g)
+    p = softmax_scores(h)
+    r = route(p, k, budget, mode, **params)
+    r["h"] = h
+    r["p"] = p
+    r["y"] = moe_ffn_combine(x_bits, r["ids"], r["w"], get_expert, tokens)
+    return r
+
+
+def expected_union_size(N: int, k: int, B: int) -> float:
+    """Closed form E[N_a] = N (1 - (1 - k/N)^B) of Sec. 1 for uniform routing."""
+    return N * (1.0 - (1.0 - k / N) ** B)
+
+
+__all__ = [n for n in dir() if not n.startswith("_")]

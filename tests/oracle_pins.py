@@ -1,0 +1,444 @@
+"""Pins of the CPU oracle to facts outside itself.
+
+Each ``check_*`` function takes the oracle module and raises AssertionError if
+the oracle disagrees with what the paper or the mathematics fixes:
+
+* the closed form E[N_a] = N(1-(1-k/N)^B) of Sec. 1, statistically, and the
+  two values the paper prints for it (golden fixture);
+* Corollary 1 (greedy is optimal for the modular objective of Eq. 2), and the
+  same for Algorithm 3's per-request step, by brute force on tiny N;
+* the balance claim of Sec. 5.1 for Algorithm 5 and the round structure of
+  its pseudocode;
+* the refinement invariants of Sec. 3.4 and the renormalised weights of
+  Sec. 2.2;
+* special cases that reduce to library routines: budget = N is plain top-k
+  (numpy lexsort), softmax / router / SwiGLU against torch float64, the
+  permutation against Python's sorted;
+* the canonical column-sum order on a hand-derived fixture, and its error
+  against the exact sum.
+
+`test_oracle_pins.py` runs them on the oracle; `test_oracle_mutations.py`
+plants mistakes in the oracle and checks that some pin fails.
+"""
+
+from __future__ import annotations
+
+import itertools
+import json
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+import torch
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+# ---------------------------------------------------------------- helpers
+
+def lexsort_top(values: np.ndarray, count: int, candidates) -> list:
+    """Top `count` candidates by (value desc, index asc) using numpy's lexsort."""
+    c = np.asarray(sorted(candidates), dtype=np.int64)
+    if count <= 0 or c.size == 0:
+        return []
+    v = np.asarray(values, dtype=np.float64)[c]
+    order = np.lexsort((c, -v))
+    return [int(x) for x in c[order][:count]]
+
+
+def exact_colsum(p: np.ndarray, rows) -> list:
+    """Exact (rational) column sums of fp32 values."""
+    rows = list(rows)
+    return [sum((Fraction(float(p[i, j])) for i in rows), Fraction(0)) for j in range(p.shape[1])]
+
+
+def quantised_scores(rng, B, N, levels=4096) -> np.ndarray:
+    """Scores that are multiples of 2^-12, so small column sums are exact in fp32."""
+    return (rng.integers(1, levels, size=(B, N)).astype(np.float64) / 4096.0).astype(np.float32)
+
+
+def distinct_colsums(p, rows) -> bool:
+    s = exact_colsum(p, rows)
+    return len(set(s)) == len(s)
+
+
+def mask_to_set(mask) -> set:
+    return {int(j) for j in np.nonzero(np.asarray(mask))[0]}
+
+
+def bf16_round(x: torch.Tensor) -> torch.Tensor:
+    return x.to(torch.bfloat16)
+
+
+def bits(t: torch.Tensor) -> np.ndarray:
+    return t.contiguous().view(torch.int16).numpy().view(np.uint16)
+
+
+# ---------------------------------------------------------------- Sec. 1
+
+def check_closed_form_golden(O):
+    with open(os.path.join(GOLDEN, "union_closed_form.json")) as f:
+        g = json.load(f)
+    for c in g["cases"]:
+        val = O.expected_union_size(c["N"], c["k"], c["B"])
+        closed = c["N"] * (1 - (1 - c["k"] / c["N"]) ** c["B"])
+        assert abs(val - closed) < 1e-9
+        assert abs(val - c["printed"]) < 0.5, (c, val)
+
+
+def check_union_statistics(O, trials=(( 64, 8, 8, 600), (256, 8, 8, 200), (256, 8, 32, 60))):
+    """Under iid continuous logits each token's top-k is a uniform k-subset, so the
+    union size of plain top-k routing has mean N(1-(1-k/N)^B) exactly (Sec. 1)."""
+    rng = np.random.default_rng(1234)
+    for N, k, B, n in trials:
+        sizes = []
+        for _ in range(n):
+            h = rng.standard_normal((B, N))
+            p = O.softmax_scores(h)
+            sizes.append(O.route(p, k, 0, O.MODE_TOPK)["union_topk"])
+        sizes = np.asarray(sizes, dtype=np.float64)
+        mean, se = sizes.mean(), sizes.std(ddof=1) / math.sqrt(n)
+        closed = N * (1 - (1 - k / N) ** B)
+        assert abs(mean - closed) <= 4 * se + 1e-9, (N, k, B, mean, closed, se)
+
+
+# ---------------------------------------------------------------- Eq. 2, Corollary 1
+
+def check_greedy_bruteforce(O, cases=40):
+    """Algorithm 2's selection maximises f(S) = sum_{j in S} sum_i g_ij over all
+    supersets of S_0 with |S| = |S_0| + min(m, N - |S_0|)."""
+    rng = np.random.default_rng(7)
+    done = 0
+    while done < cases:
+        N = int(rng.integers(4, 11))
+        B = int(rng.integers(1, 7))
+        k = int(rng.integers(1, N + 1))
+        k0 = int(rng.integers(0, 3))
+        m = int(rng.integers(0, N + 1))
+        p = quantised_scores(rng, B, N)
+        S0 = set()
+        for i in range(B):
+            S0 |= set(lexsort_top(p[i], k0, range(N)))
+        col = exact_colsum(p, range(B))
+        r = O.route(p, k, m, O.MODE_BATCH, k0=k0)
+        S = mask_to_set(r["mask"])
+        size = len(S0) + min(m, N - len(S0))
+        assert S0 <= S and len(S) == size, (S0, S, size)
+        rest = [j for j in range(N) if j not in S0]
+        best = max(sum((col[j] for j in c), Fraction(0))
+                   for c in itertools.combinations(rest, size - len(S0)))
+        got = sum((col[j] for j in S - S0), Fraction(0))
+        assert got == best, (got, best)
+        # among equal-score experts the lower index is preferred
+        for j in S - S0:
+            for q in rest:
+                if q not in S:
+                    assert col[q] < col[j] or (col[q] == col[j] and q > j), (q, j)
+        done += 1
+
+
+def check_hier_bruteforce(O, cases=25):
+    """Algorithm 3: S_r maximises the per-request proxy (Eq. 3) over supersets of
+    the request's warm-up set; Algorithm 4's batch step maximises Eq. 4 given
+    the union of the S_r."""
+    rng = np.random.default_rng(11)
+    done = 0
+    while done < cases:
+        N = int(rng.integers(4, 10))
+        T = int(rng.integers(1, 4))
+        R = int(rng.integers(1, 4))
+        B = R * T
+        k = int(rng.integers(1, N + 1))
+        k0 = int(rng.integers(0, 2))
+        m_r = int(rng.integers(0, N))
+        m = int(rng.integers(0, N))
+        p = quantised_scores(rng, B, N)
+        if not all(distinct_colsums(p, range(r * T, (r + 1) * T)) for r in range(R)):
+            continue
+        if not distinct_colsums(p, range(B)):
+            continue
+        Sb = set()
+        for r in range(R):
+            toks = range(r * T, (r + 1) * T)
+            S0r = set()
+            for i in toks:
+                S0r |= set(lexsort_top(p[i], k0, range(N)))
+            col = exact_colsum(p, toks)
+            rest = [j for j in range(N) if j not in S0r]
+            add = min(m_r, len(rest))
+            best = max(itertools.combinations(rest, add),
+                       key=lambda c: sum((col[j] for j in c), Fraction(0)))
+            Sb |= S0r | set(best)
+        col = exact_colsum(p, range(B))
+        rest = [j for j in range(N) if j not in Sb]
+        add = min(m, len(rest))
+        best = max(itertools.combinations(rest, add),
+                   key=lambda c: sum((col[j] for j in c), Fraction(0)))
+        expect = Sb | set(best)
+        r_ = O.route(p, k, m, O.MODE_HIER, k0=k0, m_r=m_r, tokens_per_request=T)
+        assert mask_to_set(r_["mask"]) == expect, (mask_to_set(r_["mask"]), expect)
+        done += 1
+
+
+def check_hier_single_request_is_batch(O, cases=20):
+    """Algorithm 4 with one request and m = 0 is Algorithm 2 with budget m_r."""
+    rng = np.random.default_rng(5)
+    for _ in range(cases):
+        N = int(rng.integers(8, 40)); B = int(rng.integers(1, 40)); k = int(rng.integers(1, 9))
+        k0 = int(rng.integers(0, 3)); m_r = int(rng.integers(0, N))
+        p = (np.exp(rng.standard_normal((B, N))) / N).astype(np.float32)
+        a = O.route(p, k, 0, O.MODE_HIER, k0=k0, m_r=m_r, tokens_per_request=B)
+        b = O.route(p, k, m_r, O.MODE_BATCH, k0=k0)
+        assert np.array_equal(a["mask"], b["mask"])
+        assert np.array_equal(a["ids"], b["ids"]) and np.array_equal(a["w"], b["w"])
+
+
+# ---------------------------------------------------------------- Sec. 5, Algorithm 5
+
+def check_group(O, cases=30):
+    """Algorithm 5/6: S_0 kept; every group that is not exhausted receives the same
+    number R of additions, its top-R remaining experts by column score; R is the
+    smallest round count reaching |S| >= m_g G (or every group is exhausted).
+    With S_0 empty, MaxLoad(S) <= ceil(|S| / G) (Sec. 5.1)."""
+    rng = np.random.default_rng(3)
+    for c in range(cases):
+        G = int(rng.choice([1, 2, 4, 8]))
+        size = int(rng.integers(1, 9))
+        N = G * size
+        B = int(rng.integers(1, 40))
+        k = int(rng.integers(1, min(N, 8) + 1))
+        k0 = 0 if c % 2 == 0 else int(rng.integers(1, 3))
+        m_g = int(rng.integers(0, size + 2))
+        p = quantised_scores(rng, B, N) if c % 3 == 0 else \
+            (np.exp(rng.standard_normal((B, N))) / N).astype(np.float32)
+        r = O.route(p, k, 0, O.MODE_GROUP, k0=k0, n_groups=G, m_g=m_g)
+        S = mask_to_set(r["mask"])
+        S0 = set()
+        for i in range(B):
+            S0 |= set(lexsort_top(p[i], k0, range(N)))
+        assert S0 <= S
+        col = np.asarray(O.canonical_column_sum(p, range(B)), dtype=np.float64)
+        avail = [[e for e in range(g * size, (g + 1) * size) if e not in S0] for g in range(G)]
+        R = 0
+        def total(R):
+            return len(S0) + sum(min(R, len(a)) for a in avail)
+        max_avail = max(len(a) for a in avail)
+        while total(R) < m_g * G and R < max_avail:
+            R += 1
+        expect = set(S0)
+        for a in avail:
+            expect |= set(lexsort_top(col, min(R, len(a)), a))
+        assert S == expect, (S, expect)
+        loads = [len([e for e in S if e // size == g]) for g in range(G)]
+        assert r["max_group_load"] == max(loads)
+        if k0 == 0:
+            assert max(loads) <= math.ceil(len(S) / G)
+
+
+# ---------------------------------------------------------------- refinement, Sec. 2.2
+
+def check_refine_invariants(O, cases=30):
+    rng = np.random.default_rng(9)
+    for c in range(cases):
+        N = int(rng.integers(2, 70)); B = int(rng.integers(1, 50)); k = int(rng.integers(1, min(N, 16) + 1))
+        mode = int(rng.integers(0, 4))
+        T = int(rng.choice([t for t in (1, 2, 4) if B % t == 0]))
+        G = int(rng.choice([g for g in (1, 2, 4) if N % g == 0]))
+        kw = dict(k0=int(rng.integers(0, 3)), m_r=int(rng.integers(0, 6)), tokens_per_request=T,
+                  n_groups=G, m_g=int(rng.integers(0, 4)))
+        ties = c % 3 == 0
+        p = (np.round(np.exp(rng.standard_normal((B, N))) * 4) / 4 / N if ties
+             else np.exp(rng.standard_normal((B, N))) / N).astype(np.float32)
+        m = int(rng.integers(0, N + 1))
+        r = O.route(p, k, m, mode, **kw)
+        S = mask_to_set(r["mask"])
+        assert r["n_selected"] == len(S)
+        kp = min(k, len(S))
+        for i in range(B):
+            ids = [int(e) for e in r["ids"][i]]
+            w = r["w"][i]
+            sel = ids[:kp]
+            assert all(e == -1 for e in ids[kp:]) and np.all(w[kp:] == 0)
+            assert len(set(sel)) == kp and set(sel) <= S
+            assert sel == lexsort_top(p[i], kp, S)
+            if kp:
+                D = sum(float(p[i, e]) for e in sel)
+                assert abs(float(np.sum(w[:kp], dtype=np.float64)) - 1.0) <= 1e-6 * max(1, kp)
+                if D > 0:
+                    ref = np.array([float(p[i, e]) / D for e in sel])
+                    assert np.allclose(w[:kp], ref, rtol=2e-6, atol=0)
+
+
+def check_zero_scores(O):
+    """A token whose scores are all zero gets equal weights 1/k'."""
+    p = np.zeros((3, 10), dtype=np.float32)
+    p[1] = np.linspace(0.1, 1.0, 10, dtype=np.float32)
+    r = O.route(p, 4, 10, O.MODE_BATCH)
+    assert list(r["ids"][0]) == [0, 1, 2, 3]
+    assert np.all(r["w"][0] == np.float32(0.25))
+    assert list(r["ids"][1]) == [9, 8, 7, 6]
+
+
+def check_budget_n_is_topk(O, cases=20):
+    """With S = E the refinement is the standard top-k routing of Sec. 2.2:
+    ids are the top-k of g_i and the weights are exp(h_i)/sum_T exp(h_j)."""
+    rng = np.random.default_rng(21)
+    for c in range(cases):
+        N = int(rng.integers(2, 80)); B = int(rng.integers(1, 40)); k = int(rng.integers(1, min(N, 16) + 1))
+        h = rng.standard_normal((B, N)) * 2
+        if c % 2:
+            h = np.round(h * 2) / 2   # many tied logits
+        p = O.softmax_scores(h)
+        k0 = int(rng.integers(0, 3))
+        rb = O.route(p, k, N, O.MODE_BATCH, k0=k0)
+        rt = O.route(p, k, 0, O.MODE_TOPK)
+        rh = O.route(p, k, 0, O.MODE_HIER, k0=k0, m_r=N, tokens_per_request=1)
+        rg = O.route(p, k, 0, O.MODE_GROUP, n_groups=1, m_g=N)
+        for r in (rb, rt, rh, rg):
+            assert r["n_selected"] == N
+            assert np.array_equal(r["ids"], rt["ids"]) and np.array_equal(r["w"], rt["w"])
+        for i in range(B):
+            ref_ids = lexsort_top(p[i], k, range(N))
+            assert [int(e) for e in rt["ids"][i]] == ref_ids
+            z = np.exp(h[i, ref_ids] - h[i, ref_ids].max())
+            ref_w = z / z.sum()
+            assert np.allclose(rt["w"][i], ref_w, rtol=3e-6, atol=1e-12)
+
+
+# ---------------------------------------------------------------- permutation
+
+def check_permutation(O, cases=20):
+    rng = np.random.default_rng(4)
+    for _ in range(cases):
+        N = int(rng.integers(1, 40)); B = int(rng.integers(1, 30)); k = int(rng.integers(1, 9))
+        ids = rng.integers(-1, N, size=(B, k)).astype(np.int32)
+        r = O.permute(ids, N)
+        pairs = sorted((int(ids[t, s]), t, s) for t in range(B) for s in range(k) if ids[t, s] >= 0)
+        assert [int(q) for q in r["perm"]] == [t * k + s for _, t, s in pairs]
+        cnt = np.bincount([e for e, _, _ in pairs], minlength=N) if pairs else np.zeros(N, int)
+        assert np.array_equal(r["counts"], cnt)
+        assert np.array_equal(r["offsets"], np.concatenate([[0], np.cumsum(cnt)]))
+        assert [int(e) for e in r["used"]] == [e for e in range(N) if cnt[e] > 0]
+
+
+# ---------------------------------------------------------------- numerics vs torch
+
+def check_router_softmax(O, cases=6):
+    g = torch.Generator().manual_seed(3)
+    for _ in range(cases):
+        B, N, d = int(torch.randint(1, 20, (1,), generator=g)), int(torch.randint(2, 70, (1,), generator=g)), 64
+        x = bf16_round(torch.randn(B, d, generator=g) * 2)
+        W = torch.randn(N, d, generator=g) / 8
+        h = O.router_logits(bits(x), W.numpy())
+        ref_h = x.to(torch.float64) @ W.to(torch.float64).T
+        assert np.allclose(h, ref_h.numpy(), rtol=1e-12, atol=1e-12)
+        p = O.softmax_scores(h)
+        ref_p = torch.softmax(ref_h, dim=1).numpy()
+        assert p.dtype == np.float32
+        assert np.allclose(p, ref_p, rtol=1.2e-7, atol=0)
+        assert np.allclose(p.astype(np.float64).sum(axis=1), 1.0, atol=N * 6e-8)
+
+
+def check_expert_ffn(O):
+    g = torch.Generator().manual_seed(8)
+    n, d, F = 5, 48, 32
+    x = bf16_round(torch.randn(n, d, generator=g))
+    Wg = bf16_round(torch.randn(F, d, generator=g) * 0.1)
+    Wu = bf16_round(torch.randn(F, d, generator=g) * 0.1)
+    Wd = bf16_round(torch.randn(d, F, generator=g) * 0.1)
+    out = O.expert_ffn(x.to(torch.float64).numpy(), bits(Wg), bits(Wu), bits(Wd))
+    X = x.to(torch.float64)
+    ref = (torch.nn.functional.silu(X @ Wg.to(torch.float64).T) * (X @ Wu.to(torch.float64).T)) \
+        @ Wd.to(torch.float64).T
+    assert np.allclose(out, ref.numpy(), rtol=1e-12, atol=1e-13)
+
+
+def check_layer_single_token(O):
+    """One token with S = E: y = sum over its top-k of g_bar_i E_i(x) (Sec. 2.1-2.2)."""
+    g = torch.Generator().manual_seed(12)
+    N, k, d, F = 12, 3, 40, 24
+    x = bf16_round(torch.randn(1, d, generator=g))
+    W_g = torch.randn(N, d, generator=g) / math.sqrt(d)
+    Wg = bf16_round(torch.randn(N, F, d, generator=g) * 0.1)
+    Wu = bf16_round(torch.randn(N, F, d, generator=g) * 0.1)
+    Wd = bf16_round(torch.randn(N, d, F, generator=g) * 0.1)
+    get = lambda e: (bits(Wg[e]), bits(Wu[e]), bits(Wd[e]))
+    r = O.moe_forward(bits(x), W_g.numpy(), get, k, 0, O.MODE_TOPK)
+    X = x.to(torch.float64)
+    h = X @ W_g.to(torch.float64).T
+    val, idx = torch.topk(h[0], k)
+    gbar = torch.softmax(val, dim=0)
+    y = torch.zeros(d, dtype=torch.float64)
+    for wgt, e in zip(gbar, idx):
+        a = torch.nn.functional.silu(X[0] @ Wg[e].to(torch.float64).T) * (X[0] @ Wu[e].to(torch.float64).T)
+        y += wgt * (a @ Wd[e].to(torch.float64).T)
+    assert [int(e) for e in r["ids"][0]] == [int(e) for e in idx]
+    assert np.allclose(r["y"][0], y.numpy(), rtol=1e-5, atol=1e-7 * float(y.abs().max()))
+
+
+def check_combine_multi_token(O):
+    """y for several tokens equals per-token sums of w * E_e(x) (Sec. 2.1) computed
+    with torch, for a routing with padding slots."""
+    g = torch.Generator().manual_seed(13)
+    N, k, d, F, B = 6, 3, 16, 8, 4
+    x = bf16_round(torch.randn(B, d, generator=g))
+    Wg = bf16_round(torch.randn(N, F, d, generator=g) * 0.2)
+    Wu = bf16_round(torch.randn(N, F, d, generator=g) * 0.2)
+    Wd = bf16_round(torch.randn(N, d, F, generator=g) * 0.2)
+    ids = np.array([[0, 3, -1], [5, 0, 1], [2, -1, -1], [4, 5, 3]], dtype=np.int32)
+    w = np.array([[0.7, 0.3, 0], [0.5, 0.25, 0.25], [1, 0, 0], [0.2, 0.3, 0.5]], dtype=np.float32)
+    get = lambda e: (bits(Wg[e]), bits(Wu[e]), bits(Wd[e]))
+    y = O.moe_ffn_combine(bits(x), ids, w, get)
+    X = x.to(torch.float64)
+    for t in range(B):
+        ref = torch.zeros(d, dtype=torch.float64)
+        for s in range(k):
+            e = int(ids[t, s])
+            if e < 0:
+                continue
+            a = torch.nn.functional.silu(X[t] @ Wg[e].to(torch.float64).T) * (X[t] @ Wu[e].to(torch.float64).T)
+            ref += float(w[t, s]) * (a @ Wd[e].to(torch.float64).T)
+        assert np.allclose(y[t], ref.numpy(), rtol=1e-12, atol=1e-14)
+    sub = O.moe_ffn_combine(bits(x), ids, w, get, tokens=[3, 1])
+    assert np.allclose(sub, y[[3, 1]], rtol=1e-12, atol=1e-14)
+
+
+# ---------------------------------------------------------------- canonical column sum
+
+def check_canonical_sum_golden(O):
+    with open(os.path.join(GOLDEN, "canonical_sum.json")) as f:
+        g = json.load(f)
+    for col in g["columns"]:
+        rows = np.zeros((col["rows"], 1), dtype=np.uint32)
+        for key, val in col["rows_hex"].items():
+            lo, _, hi = key.partition("-")
+            rows[int(lo):int(hi or lo) + 1] = int(val, 16)
+        p = rows.view(np.float32)
+        got = O.canonical_column_sum(p, range(col["rows"])).view(np.uint32)[0]
+        assert int(got) == int(col["expected_hex"], 16), (col["describe"], hex(int(got)))
+
+
+def check_canonical_sum_bound(O, cases=20):
+    """|canonical - exact| <= (5 + chunks) u sum|p|, u = 2^-24 (depth-5 tree per
+    chunk plus one accumulation per chunk)."""
+    rng = np.random.default_rng(17)
+    for _ in range(cases):
+        B = int(rng.integers(1, 150)); N = int(rng.integers(1, 10))
+        p = (np.exp(rng.standard_normal((B, N)) * 3) / N).astype(np.float32)
+        rows = list(rng.permutation(B)) if rng.integers(2) else list(range(B))
+        got = O.canonical_column_sum(p, rows)
+        ex = exact_colsum(p, rows)
+        chunks = (len(rows) + 31) // 32
+        for j in range(N):
+            bound = (5 + chunks) * 2.0 ** -24 * float(ex[j]) * 1.0000001
+            assert abs(Fraction(float(got[j])) - ex[j]) <= Fraction(bound), (B, j)
+
+
+ALL_CHECKS = [
+    check_closed_form_golden, check_union_statistics, check_greedy_bruteforce,
+    check_hier_bruteforce, check_hier_single_request_is_batch, check_group,
+    check_refine_invariants, check_zero_scores, check_budget_n_is_topk, check_permutation,
+    check_router_softmax, check_expert_ffn, check_layer_single_token,
+    check_combine_multi_token, check_canonical_sum_golden, check_canonical_sum_bound,
+]
