@@ -1,0 +1,183 @@
+/*
+ * xshare.h — C ABI of libxshare.so: one XShare MoE-layer forward on one GPU.
+ *
+ * XShare (arxiv 2602.07265) restricts a decode / verify batch to a set S of
+ * experts chosen for the batch as a whole, by maximising the total gating
+ * score of S under an expert budget (Sec. 3.2, Eq. 2), and then routes every
+ * token to its top-k experts inside S (Sec. 3.4, refinement).
+ *
+ * Conventions for every entry point
+ *   - Device pointers point to memory of the current CUDA device, row-major and
+ *     contiguous, at least 16-byte aligned unless stated otherwise.  bf16
+ *     tensors are passed as uint16_t (the raw bf16 bit pattern).
+ *   - The caller owns every buffer.  The library allocates nothing: scratch
+ *     space is the caller's `workspace` of at least xshare_workspace_size()
+ *     bytes, 256-byte aligned, which the calls overwrite.
+ *   - Calls are asynchronous and stream-ordered on `stream` (a cudaStream_t;
+ *     NULL is the legacy default stream).  No call synchronises the stream or
+ *     the device.  Two calls that share a workspace must not overlap.
+ *   - Invalid arguments are detected on the host before anything is launched
+ *     and returned as a negative XS_ERR_* code; nothing is written then.
+ *     A failed kernel launch returns XS_ERR_CUDA.  A device-side failure (a
+ *     bounded wait that ran out) is reported in xs_stats.status, which the
+ *     caller reads after synchronising.
+ *   - Scores must be finite (no NaN): selection compares them as fp32 values.
+ *
+ * Limits: 1 <= N <= 1024 experts; 1 <= k <= min(N, 16); 0 <= k0 <= min(N, 16);
+ * 1 <= B <= 8192 tokens; for xshare_moe_forward d % 128 == 0 and F % 128 == 0.
+ */
+#ifndef XSHARE_H
+#define XSHARE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+struct CUstream_st;
+/* A cudaStream_t. */
+typedef struct CUstream_st *xs_stream_t;
+
+/* Selection modes.
+ *   XS_MODE_TOPK : S = E, plain top-k routing (the paper's baseline, Sec. 2.2).
+ *   XS_MODE_BATCH: Algorithm 2 — warm-up S_0 = union of per-token Top k0, then
+ *                  GreedySelect (Algorithm 1 with a fixed budget): the `budget`
+ *                  experts of E \ S_0 with the largest column score
+ *                  scores[j] = sum_i g_ij are added (Sec. 3.4).
+ *   XS_MODE_GROUP: Algorithm 6 — warm-up S_0, then Algorithm 5: full rounds over
+ *                  the G contiguous expert groups, each round adding every
+ *                  non-exhausted group's best remaining expert, until
+ *                  |S| >= m_g * G (Sec. 5, Eq. 5).
+ *   XS_MODE_HIER : Algorithm 4 — per request (contiguous runs of
+ *                  tokens_per_request tokens) Algorithm 3:
+ *                  S_r = S0_r + Top m_r of the request's column scores; then
+ *                  S = union S_r plus the `budget` best remaining experts by the
+ *                  batch column score (Sec. 4, Eq. 3-4).
+ * Ordering everywhere: larger score first, equal scores -> lower expert index.
+ * Column scores are fp32 sums in a fixed order: rows in chunks of 32 (last one
+ * zero-padded), a halving tree v[l] += v[l+o], o = 16, 8, 4, 2, 1, inside a
+ * chunk, chunk sums added left to right from 0. */
+enum {
+  XS_MODE_TOPK = 0,
+  XS_MODE_BATCH = 1,
+  XS_MODE_GROUP = 2,
+  XS_MODE_HIER = 3
+};
+
+/* Selection parameters (fields a mode does not use are ignored). */
+typedef struct {
+  int32_t k0;                 /* warm-up: Top k0 per token (Algorithms 2, 3, 6); 0 = none */
+  int32_t m_r;                /* HIER: per-request budget m_r (Algorithm 3) */
+  int32_t tokens_per_request; /* HIER: 1 + L_s (Sec. 4.1); B % tokens_per_request == 0 */
+  int32_t n_groups;           /* GROUP: G (Sec. 5); N % G == 0.  Also used by the
+                                 max_group_load statistic in every mode; 0 = 1 */
+  int32_t m_g;                /* GROUP: per-group budget m_g (Algorithm 5) */
+} xs_route_params;
+
+/* Per-call statistics, written by the device into caller memory. */
+typedef struct {
+  int32_t n_selected;     /* |S| */
+  int32_t n_used;         /* |U|: experts with at least one routed (token, slot) */
+  int32_t union_topk;     /* |union_i Top k(G_i, E)|: experts plain top-k would activate */
+  int32_t max_group_load; /* max_g |S intersect E_g| over n_groups groups (Sec. 5.1) */
+  int32_t n_pairs;        /* routed (token, slot) pairs = B * min(k, |S|) */
+  int32_t status;         /* 0, or an XS_DEV_* code */
+  int32_t reserved[2];
+} xs_stats;
+
+/* Host-side error codes (return values). */
+#define XS_OK 0
+#define XS_ERR_SHAPE (-1)     /* B, N, k, d or F out of range or misaligned */
+#define XS_ERR_PARAM (-2)     /* mode, budget, k0, m_r, m_g, n_groups or tokens_per_request invalid */
+#define XS_ERR_NULL (-3)      /* a required pointer is NULL */
+#define XS_ERR_WORKSPACE (-4) /* workspace NULL, too small or not 256-byte aligned */
+#define XS_ERR_ALIGN (-5)     /* a tensor pointer is not 16-byte aligned */
+#define XS_ERR_CUDA (-6)      /* a CUDA runtime / launch error */
+#define XS_ERR_DEVICE (-7)    /* the current device is not an sm_103 (GB300) GPU */
+
+/* Device-side status codes (xs_stats.status). */
+#define XS_DEV_OK 0
+#define XS_DEV_TIMEOUT 1      /* a bounded wait inside a kernel ran out */
+
+/* Bytes of workspace the calls below need for these sizes.  For
+ * xshare_route pass d = F = 0.  Returns 0 for arguments the calls would
+ * reject.  Depends on the current device's SM count. */
+size_t xshare_workspace_size(int B, int N, int k, int d, int F, int mode,
+                             const xs_route_params *prm);
+
+/* Steps a3-a7 of the path: batch-aware selection and refinement on given scores.
+ *
+ *   scores   [B, N] fp32, device: gating scores g_ij (e.g. the dense softmax
+ *            of the router logits, Sec. 2.2).
+ *   budget   m: experts the greedy step adds beyond the warm-up set
+ *            (BATCH, HIER); ignored by TOPK and GROUP.
+ *   sel_mask [N] uint8, device, out: 1 for experts in S.
+ *   topk_ids [B, k] int32, device, out: per token the min(k, |S|) best experts
+ *            of S, best first (Top k(G_i, S), Algorithms 2, 4, 6); unused slots -1.
+ *   topk_w   [B, k] fp32, device, out: renormalised weights
+ *            g_ie / D_i, D_i = fp32 sum of the routed scores in slot order
+ *            (Sec. 2.2 restricted to the routed set); unused slots 0.  If
+ *            D_i == 0 every routed weight is 1/min(k, |S|).
+ *   stats    xs_stats, device, out, nullable.
+ *   expert_counts  [N] int32, device, out, nullable: pairs routed per expert.
+ *   expert_offsets [N + 1] int32, device, out, nullable: exclusive prefix sum.
+ *   perm     [B * k] int32, device, out, nullable: pair ids t * k + slot grouped
+ *            by expert (ascending), ascending inside an expert; the first
+ *            stats.n_pairs entries are written.
+ */
+int xshare_route(const float *scores, int B, int N, int k, int budget, int mode,
+                 const xs_route_params *prm, uint8_t *sel_mask, int32_t *topk_ids,
+                 float *topk_w, xs_stats *stats, int32_t *expert_counts,
+                 int32_t *expert_offsets, int32_t *perm, void *workspace,
+                 size_t ws_bytes, xs_stream_t stream);
+
+/* The whole path a1-a9: one MoE layer forward, routed part (Sec. 2.1).
+ *
+ *   x       [B, d] bf16, device: token hidden states.
+ *   W_g     [N, d] fp32, device: router weights; h = W_g x (Sec. 2.2).
+ *   W_gate  [N, F, d] bf16, device; W_up [N, F, d] bf16; W_down [N, d, F] bf16:
+ *           expert e computes E_e(x) = W_down[e] (silu(W_gate[e] x) * (W_up[e] x)).
+ *           Only the experts that receive a token are read.
+ *   y       [B, d] bf16, device, out: y_t = sum over slots of w_ts E_{ids_ts}(x_t),
+ *           accumulated in fp32 and rounded once to bf16.
+ *   scores_out [B, N] fp32, device, out, nullable: the dense softmax scores g.
+ *   sel_mask, topk_ids, topk_w, stats: as in xshare_route, each nullable.
+ * Other arguments as in xshare_route.
+ */
+int xshare_moe_forward(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
+                       const uint16_t *W_up, const uint16_t *W_down, int B, int d, int F,
+                       int N, int k, int budget, int mode, const xs_route_params *prm,
+                       uint16_t *y, float *scores_out, uint8_t *sel_mask,
+                       int32_t *topk_ids, float *topk_w, xs_stats *stats, void *workspace,
+                       size_t ws_bytes, xs_stream_t stream);
+
+/* Kernel stages of xshare_moe_forward, in launch order. */
+#define XS_N_STAGES 6
+
+/* xshare_moe_forward that also records CUDA events on `stream` between its
+ * kernel launches, so a caller can time each stage on the launching stream:
+ * stage_events[0] before the first launch and stage_events[i + 1] after
+ * stage i, for i < XS_N_STAGES.  stage_events is a host array of
+ * XS_N_STAGES + 1 cudaEvent_t created by the caller (not NULL).  Results are
+ * identical to xshare_moe_forward. */
+int xshare_moe_forward_profiled(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
+                                const uint16_t *W_up, const uint16_t *W_down, int B, int d,
+                                int F, int N, int k, int budget, int mode,
+                                const xs_route_params *prm, uint16_t *y, float *scores_out,
+                                uint8_t *sel_mask, int32_t *topk_ids, float *topk_w,
+                                xs_stats *stats, void *workspace, size_t ws_bytes,
+                                xs_stream_t stream, void *const *stage_events);
+
+/* Name of stage i of xshare_moe_forward (e.g. "router"), or "" if out of range. */
+const char *xshare_stage_name(int i);
+
+/* A static string describing an XS_ERR_* or XS_DEV_* code (never NULL). */
+const char *xshare_strerror(int code);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* XSHARE_H */

@@ -1,0 +1,299 @@
+// C ABI of libxshare.so (include/xshare.h): argument checks, workspace plan
+// and the stream-ordered launch sequence of the MoE-layer forward.
+#include <cuda_runtime.h>
+
+#include <cstdint>
+#include <cstring>
+
+#include "xs_internal.cuh"
+
+namespace xs {
+namespace {
+
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
+
+struct DevInfo {
+  int known;
+  int ok;
+  int n_sms;
+};
+DevInfo g_dev[64];
+
+// The current device's SM count, or a negative XS_ERR code.
+int current_device_sms() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return XS_ERR_CUDA;
+  DevInfo &di = g_dev[dev];
+  if (!di.known) {
+    int major = 0, minor = 0, sms = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return XS_ERR_CUDA;
+    di.ok = (major == 10 && minor == 3);
+    di.n_sms = sms;
+    di.known = 1;
+  }
+  return di.ok ? di.n_sms : XS_ERR_DEVICE;
+}
+
+int check_route_args(int B, int N, int k, int budget, int mode, const xs_route_params *prm) {
+  if (prm == nullptr) return XS_ERR_NULL;
+  if (B < 1 || B > kMaxB || N < 1 || N > kMaxN || k < 1 || k > kMaxK || k > N) return XS_ERR_SHAPE;
+  if (mode < XS_MODE_TOPK || mode > XS_MODE_HIER) return XS_ERR_PARAM;
+  if (budget < 0 || prm->k0 < 0 || prm->k0 > kMaxK || prm->k0 > N || prm->m_r < 0 || prm->m_g < 0 ||
+      prm->n_groups < 0)
+    return XS_ERR_PARAM;
+  if (prm->n_groups > 0 && (prm->n_groups > N || N % prm->n_groups != 0)) return XS_ERR_PARAM;
+  if (mode == XS_MODE_GROUP && prm->n_groups < 1) return XS_ERR_PARAM;
+  if (mode == XS_MODE_HIER &&
+      (prm->tokens_per_request < 1 || prm->tokens_per_request > B || B % prm->tokens_per_request != 0))
+    return XS_ERR_PARAM;
+  return XS_OK;
+}
+
+int check_ffn_shape(int d, int F) {
+  if (d < 128 || F < 128 || d % 128 != 0 || F % 128 != 0) return XS_ERR_SHAPE;
+  if ((long long)d > (1 << 20) || (long long)F > (1 << 20)) return XS_ERR_SHAPE;
+  return XS_OK;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+template <class T>
+T *at(void *ws, size_t off) {
+  return reinterpret_cast<T *>(static_cast<char *>(ws) + off);
+}
+
+RouteArgs route_args(const Plan &pl, void *ws, int B, int N, int k, int budget, int mode,
+                     const xs_route_params *prm) {
+  RouteArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.B = B;
+  a.N = N;
+  a.k = k;
+  a.budget = budget;
+  a.mode = mode;
+  a.k0 = (mode == XS_MODE_TOPK) ? 0 : prm->k0;
+  a.m_r = prm->m_r;
+  a.T = prm->tokens_per_request < 1 ? 1 : prm->tokens_per_request;
+  a.G = prm->n_groups < 1 ? 1 : prm->n_groups;
+  a.m_g = prm->m_g > N ? N : prm->m_g;
+  a.p = at<float>(ws, pl.p);
+  a.mask = at<uint8_t>(ws, pl.mask);
+  a.ids = at<int32_t>(ws, pl.ids);
+  a.w = at<float>(ws, pl.w);
+  a.toptok = at<int32_t>(ws, pl.toptok);
+  a.counts = at<int32_t>(ws, pl.counts);
+  a.offsets = at<int32_t>(ws, pl.offsets);
+  a.perm = at<int32_t>(ws, pl.perm);
+  a.pos = at<int32_t>(ws, pl.pos);
+  a.tiles = at<Tile>(ws, pl.tiles);
+  a.meta = at<Meta>(ws, pl.meta);
+  return a;
+}
+
+}  // namespace
+
+Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms) {
+  Plan pl;
+  std::memset(&pl, 0, sizeof(pl));
+  pl.n_sms = n_sms;
+  pl.max_pairs = B * k;
+  pl.max_tiles = N + (B * k) / kTileTok + 1;
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    size_t r = o;
+    o = align_up(o + bytes);
+    return r;
+  };
+  pl.h = take((size_t)B * N * 4);
+  pl.p = take((size_t)B * N * 4);
+  pl.mask = take((size_t)N);
+  pl.ids = take((size_t)B * k * 4);
+  pl.w = take((size_t)B * k * 4);
+  pl.toptok = take((size_t)B * kMaxK * 4);
+  pl.counts = take((size_t)N * 4);
+  pl.offsets = take((size_t)(N + 1) * 4);
+  pl.perm = take((size_t)B * k * 4);
+  pl.pos = take((size_t)B * k * 4);
+  pl.tiles = take((size_t)pl.max_tiles * sizeof(Tile));
+  pl.meta = take(sizeof(Meta));
+  if (with_ffn) {
+    pl.xp = take((size_t)pl.max_pairs * d * 2);
+    pl.act = take((size_t)pl.max_pairs * F * 2);
+    pl.out = take((size_t)pl.max_pairs * d * 4);
+    pl.ffn_part = take(ffn_part_bytes(n_sms));
+    pl.ffn_cnt = take(ffn_cnt_words(pl.max_tiles, d, F) * 4);
+  }
+  pl.total = o;
+  return pl;
+}
+
+}  // namespace xs
+
+using namespace xs;
+
+extern "C" size_t xshare_workspace_size(int B, int N, int k, int d, int F, int mode,
+                                        const xs_route_params *prm) {
+  if (check_route_args(B, N, k, 0, mode, prm) != XS_OK) return 0;
+  const bool ffn = (d != 0 || F != 0);
+  if (ffn && check_ffn_shape(d, F) != XS_OK) return 0;
+  const int sms = current_device_sms();
+  if (sms < 0) return 0;
+  return make_plan(B, N, k, d, F, ffn, sms).total;
+}
+
+extern "C" int xshare_route(const float *scores, int B, int N, int k, int budget, int mode,
+                            const xs_route_params *prm, uint8_t *sel_mask, int32_t *topk_ids,
+                            float *topk_w, xs_stats *stats, int32_t *expert_counts,
+                            int32_t *expert_offsets, int32_t *perm, void *workspace,
+                            size_t ws_bytes, xs_stream_t stream) {
+  int rc = check_route_args(B, N, k, budget, mode, prm);
+  if (rc != XS_OK) return rc;
+  if (!scores || !sel_mask || !topk_ids || !topk_w) return XS_ERR_NULL;
+  if (!aligned16(scores)) return XS_ERR_ALIGN;
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return XS_ERR_WORKSPACE;
+  const int sms = current_device_sms();
+  if (sms < 0) return sms;
+  const Plan pl = make_plan(B, N, k, 0, 0, false, sms);
+  if (ws_bytes < pl.total) return XS_ERR_WORKSPACE;
+  RouteArgs a = route_args(pl, workspace, B, N, k, budget, mode, prm);
+  a.p = const_cast<float *>(scores);  // read only when logits == nullptr
+  a.mask = sel_mask;
+  a.ids = topk_ids;
+  a.w = topk_w;
+  a.stats = stats;
+  a.counts_out = expert_counts;
+  a.offsets_out = expert_offsets;
+  a.perm_out = perm;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return launch_route(a, s) == cudaSuccess ? XS_OK : XS_ERR_CUDA;
+}
+
+namespace {
+
+const char *const kStageNames[XS_N_STAGES] = {"router", "select", "gather", "ffn_gate_up",
+                                              "ffn_down", "combine"};
+
+int forward_impl(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
+                 const uint16_t *W_up, const uint16_t *W_down, int B, int d, int F, int N, int k,
+                 int budget, int mode, const xs_route_params *prm, uint16_t *y,
+                 float *scores_out, uint8_t *sel_mask, int32_t *topk_ids, float *topk_w,
+                 xs_stats *stats, void *workspace, size_t ws_bytes, xs_stream_t stream,
+                 void *const *events) {
+  int rc = check_route_args(B, N, k, budget, mode, prm);
+  if (rc != XS_OK) return rc;
+  rc = check_ffn_shape(d, F);
+  if (rc != XS_OK) return rc;
+  if (!x || !W_g || !W_gate || !W_up || !W_down || !y) return XS_ERR_NULL;
+  if (!aligned16(x) || !aligned16(W_g) || !aligned16(W_gate) || !aligned16(W_up) ||
+      !aligned16(W_down) || !aligned16(y) || (scores_out && !aligned16(scores_out)))
+    return XS_ERR_ALIGN;
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return XS_ERR_WORKSPACE;
+  const int sms = current_device_sms();
+  if (sms < 0) return sms;
+  const Plan pl = make_plan(B, N, k, d, F, true, sms);
+  if (ws_bytes < pl.total) return XS_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+
+  RouteArgs a = route_args(pl, workspace, B, N, k, budget, mode, prm);
+  float *h = at<float>(workspace, pl.h);
+  a.logits = h;
+  if (scores_out) a.p = scores_out;
+  if (sel_mask) a.mask = sel_mask;
+  if (topk_ids) a.ids = topk_ids;
+  if (topk_w) a.w = topk_w;
+  a.stats = stats;
+  a.zero_words = at<int32_t>(workspace, pl.ffn_cnt);
+  a.zero_count = (int)ffn_cnt_words(pl.max_tiles, d, F);
+
+  FfnArgs f;
+  std::memset(&f, 0, sizeof(f));
+  f.W_gate = W_gate;
+  f.W_up = W_up;
+  f.W_down = W_down;
+  f.xp = at<uint16_t>(workspace, pl.xp);
+  f.act = at<uint16_t>(workspace, pl.act);
+  f.out = at<float>(workspace, pl.out);
+  f.tiles = a.tiles;
+  f.meta = a.meta;
+  f.stats = stats;
+  f.part = at<void>(workspace, pl.ffn_part);
+  f.cnt = at<int32_t>(workspace, pl.ffn_cnt);
+  f.N = N;
+  f.d = d;
+  f.F = F;
+  f.max_pairs = pl.max_pairs;
+  f.max_tiles = pl.max_tiles;
+  f.n_sms = sms;
+
+  auto mark = [&](int i) {
+    return events == nullptr ||
+           cudaEventRecord(reinterpret_cast<cudaEvent_t>(events[i]), s) == cudaSuccess;
+  };
+  if (!mark(0)) return XS_ERR_CUDA;
+  if (launch_router_logits(x, W_g, h, B, N, d, s) != cudaSuccess || !mark(1)) return XS_ERR_CUDA;
+  if (launch_route(a, s) != cudaSuccess || !mark(2)) return XS_ERR_CUDA;
+  if (launch_gather(x, a.perm, a.meta, const_cast<uint16_t *>(f.xp), pl.max_pairs, d, k, s) !=
+          cudaSuccess ||
+      !mark(3))
+    return XS_ERR_CUDA;
+  if (launch_ffn_gate_up(f, s) != cudaSuccess || !mark(4)) return XS_ERR_CUDA;
+  if (launch_ffn_down(f, s) != cudaSuccess || !mark(5)) return XS_ERR_CUDA;
+  if (launch_combine(f.out, a.pos, a.w, a.meta, y, B, d, k, s) != cudaSuccess || !mark(6))
+    return XS_ERR_CUDA;
+  return XS_OK;
+}
+
+}  // namespace
+
+extern "C" int xshare_moe_forward(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
+                                  const uint16_t *W_up, const uint16_t *W_down, int B, int d,
+                                  int F, int N, int k, int budget, int mode,
+                                  const xs_route_params *prm, uint16_t *y, float *scores_out,
+                                  uint8_t *sel_mask, int32_t *topk_ids, float *topk_w,
+                                  xs_stats *stats, void *workspace, size_t ws_bytes,
+                                  xs_stream_t stream) {
+  return forward_impl(x, W_g, W_gate, W_up, W_down, B, d, F, N, k, budget, mode, prm, y,
+                      scores_out, sel_mask, topk_ids, topk_w, stats, workspace, ws_bytes, stream,
+                      nullptr);
+}
+
+extern "C" int xshare_moe_forward_profiled(const uint16_t *x, const float *W_g,
+                                           const uint16_t *W_gate, const uint16_t *W_up,
+                                           const uint16_t *W_down, int B, int d, int F, int N,
+                                           int k, int budget, int mode,
+                                           const xs_route_params *prm, uint16_t *y,
+                                           float *scores_out, uint8_t *sel_mask,
+                                           int32_t *topk_ids, float *topk_w, xs_stats *stats,
+                                           void *workspace, size_t ws_bytes, xs_stream_t stream,
+                                           void *const *stage_events) {
+  if (stage_events == nullptr) return XS_ERR_NULL;
+  for (int i = 0; i <= XS_N_STAGES; ++i)
+    if (stage_events[i] == nullptr) return XS_ERR_NULL;
+  return forward_impl(x, W_g, W_gate, W_up, W_down, B, d, F, N, k, budget, mode, prm, y,
+                      scores_out, sel_mask, topk_ids, topk_w, stats, workspace, ws_bytes, stream,
+                      stage_events);
+}
+
+extern "C" const char *xshare_stage_name(int i) {
+  return (i >= 0 && i < XS_N_STAGES) ? kStageNames[i] : "";
+}
+
+extern "C" const char *xshare_strerror(int code) {
+  switch (code) {
+    case XS_OK: return "ok";
+    case XS_ERR_SHAPE: return "shape out of range (B, N, k, d or F) or d/F not a multiple of 128";
+    case XS_ERR_PARAM: return "invalid selection parameter (mode, budget, k0, m_r, m_g, n_groups or tokens_per_request)";
+    case XS_ERR_NULL: return "a required pointer is NULL";
+    case XS_ERR_WORKSPACE: return "workspace NULL, too small or not 256-byte aligned";
+    case XS_ERR_ALIGN: return "a tensor pointer is not 16-byte aligned";
+    case XS_ERR_CUDA: return "CUDA runtime or launch error";
+    case XS_ERR_DEVICE: return "the current device is not an sm_103 (GB300) GPU";
+    case XS_DEV_TIMEOUT: return "device: a bounded wait inside a kernel ran out";
+    default: return "unknown xshare error code";
+  }
+}

@@ -1,0 +1,100 @@
+// Internal declarations shared by the translation units of libxshare.so.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cstddef>
+#include <cstdint>
+
+#include "xshare.h"
+
+namespace xs {
+
+constexpr int kMaxN = 1024;     // experts
+constexpr int kMaxK = 16;       // top-k and warm-up k0
+constexpr int kMaxB = 8192;     // tokens
+constexpr int kTileTok = 128;   // tokens of one expert handled by one FFN tile
+constexpr int kRouteThreads = 1024;
+
+// One FFN work tile: up to kTileTok consecutive rows of the permuted pair
+// list, all routed to `expert`.
+struct Tile {
+  int32_t expert;
+  int32_t row0;
+  int32_t ntok;
+  int32_t pad;
+};
+
+// Device-side facts of one call, written by the routing kernel and read by
+// the kernels after it (so that no host synchronisation is needed).
+struct Meta {
+  int32_t n_pairs;      // B * k'
+  int32_t n_tiles;      // FFN tiles
+  int32_t kprime;       // k' = min(k, |S|)
+  int32_t n_selected;
+  int32_t n_used;
+  int32_t union_topk;
+  int32_t max_group_load;
+  int32_t status;       // XS_DEV_*
+  int32_t pad[8];
+};
+
+// Byte offsets of every workspace region (256-byte aligned).
+struct Plan {
+  size_t h, p, mask, ids, w, toptok, counts, offsets, perm, pos, tiles, meta;
+  size_t xp, act, out, ffn_part, ffn_cnt;
+  size_t total;
+  int max_pairs, max_tiles, n_sms;
+};
+
+Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms);
+
+struct RouteArgs {
+  const float *logits;   // nullable: if set, p = softmax(logits) is computed first
+  float *p;              // [B, N] scores (input if logits == nullptr, else output)
+  int B, N, k, budget, mode, k0, m_r, T, G, m_g;
+  uint8_t *mask;         // [N]
+  int32_t *ids;          // [B, k]
+  float *w;              // [B, k]
+  int32_t *toptok;       // [B, 16] per-token ranked top over E
+  int32_t *counts;       // [N]
+  int32_t *offsets;      // [N + 1]
+  int32_t *perm;         // [B * k]
+  int32_t *pos;          // [B * k] inverse of perm (row of pair t*k+s), -1 if unrouted
+  Tile *tiles;           // [max_tiles]
+  Meta *meta;
+  xs_stats *stats;       // nullable
+  int32_t *counts_out;   // nullable caller copies
+  int32_t *offsets_out;
+  int32_t *perm_out;
+  int32_t *zero_words;   // nullable: region cleared for the FFN kernels
+  int zero_count;
+};
+
+cudaError_t launch_route(const RouteArgs &a, cudaStream_t s);
+cudaError_t launch_router_logits(const uint16_t *x, const float *Wg, float *h, int B, int N,
+                                 int d, cudaStream_t s);
+cudaError_t launch_gather(const uint16_t *x, const int32_t *perm, const Meta *meta,
+                          uint16_t *xp, int max_pairs, int d, int k, cudaStream_t s);
+cudaError_t launch_combine(const float *out, const int32_t *pos, const float *w,
+                           const Meta *meta, uint16_t *y, int B, int d, int k,
+                           cudaStream_t s);
+
+struct FfnArgs {
+  const uint16_t *W_gate, *W_up, *W_down;
+  const uint16_t *xp;    // [max_pairs, d] permuted token rows
+  uint16_t *act;         // [max_pairs, F] silu(g) * u, bf16
+  float *out;            // [max_pairs, d] expert outputs, fp32
+  const Tile *tiles;
+  Meta *meta;
+  xs_stats *stats;       // nullable
+  void *part;            // partial-sum scratch
+  int32_t *cnt;          // arrival counters (cleared by the routing kernel)
+  int N, d, F, max_pairs, max_tiles, n_sms;
+};
+
+cudaError_t launch_ffn_gate_up(const FfnArgs &a, cudaStream_t s);
+cudaError_t launch_ffn_down(const FfnArgs &a, cudaStream_t s);
+size_t ffn_part_bytes(int n_sms);
+size_t ffn_cnt_words(int max_tiles, int d, int F);
+
+}  // namespace xs

@@ -26,6 +26,7 @@ import numpy as np
 import torch
 
 MODE_TOPK, MODE_BATCH, MODE_GROUP, MODE_HIER = 0, 1, 2, 3
+MODES = {"topk": MODE_TOPK, "batch": MODE_BATCH, "group": MODE_GROUP, "hier": MODE_HIER}
 
 EXPERT_STD = 0.02
 
@@ -124,21 +125,25 @@ def batch_stream(w: Workload, seed: int, count: int) -> list:
 
 
 def expert_weights(w: Workload, seed: int = 0, device: str = "cuda",
-                   experts: Optional[list] = None) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+                   experts: Optional[list] = None,
+                   f_rows: Optional[int] = None) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
     """W_gate [N, F, d], W_up [N, F, d], W_down [N, d, F], bf16, N(0, 0.02).
 
     Drawn expert by expert from a generator on `device`, so that peak
     temporary memory stays at one fp32 expert matrix.  With `experts` given
     (CPU only), only those experts are drawn and the tensors are
     [len(experts), ...]; each expert's values then depend on (seed, e) only.
+    With `f_rows` (CPU only) only the first f_rows hidden units are drawn
+    (W_gate, W_up [., f_rows, d], W_down [., d, f_rows]).
     """
-    N, F, d = w.N, w.F, w.d
+    N, d = w.N, w.d
+    F = w.F if f_rows is None else int(f_rows)
     ids = list(range(N)) if experts is None else list(experts)
     n = len(ids)
     Wg = torch.empty(n, F, d, dtype=torch.bfloat16, device=device)
     Wu = torch.empty(n, F, d, dtype=torch.bfloat16, device=device)
     Wd = torch.empty(n, d, F, dtype=torch.bfloat16, device=device)
-    if device == "cpu" or experts is not None:
+    if device == "cpu" or experts is not None or f_rows is not None:
         for i, e in enumerate(ids):
             g = _gen(seed, 1000 + e)
             for t, shape in ((Wg, (F, d)), (Wu, (F, d)), (Wd, (d, F))):

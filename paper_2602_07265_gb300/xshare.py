@@ -1,0 +1,175 @@
+"""ctypes binding of libxshare.so (include/xshare.h).
+
+Argument marshalling only: each function checks tensor devices, dtypes and
+contiguity, passes raw pointers and the current CUDA stream to the C ABI and
+raises `XShareError` on a non-zero return code.  Every step of the layer runs
+in the library's CUDA kernels; there is no other code path.  Importing this
+module loads the library and raises if it has not been built.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import torch
+
+from . import _build
+
+MODE_TOPK, MODE_BATCH, MODE_GROUP, MODE_HIER = 0, 1, 2, 3
+MODES = {"topk": MODE_TOPK, "batch": MODE_BATCH, "group": MODE_GROUP, "hier": MODE_HIER}
+
+XS_DEV_OK, XS_DEV_TIMEOUT = 0, 1
+STATS_FIELDS = ("n_selected", "n_used", "union_topk", "max_group_load", "n_pairs", "status")
+STATS_WORDS = 8
+
+
+class XShareError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: xshare error {code}: {xshare_strerror(code)}")
+
+
+class RouteParams(ctypes.Structure):
+    """xs_route_params."""
+    _fields_ = [("k0", ctypes.c_int32), ("m_r", ctypes.c_int32),
+                ("tokens_per_request", ctypes.c_int32), ("n_groups", ctypes.c_int32),
+                ("m_g", ctypes.c_int32)]
+
+
+def route_params(k0: int = 0, m_r: int = 0, tokens_per_request: int = 1, n_groups: int = 1,
+                 m_g: int = 0) -> RouteParams:
+    return RouteParams(k0, m_r, tokens_per_request, n_groups, m_g)
+
+
+def _load() -> ctypes.CDLL:
+    path = _build.LIB
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with __graft_entry__.build() "
+                           "(there is no fallback implementation)")
+    lib = ctypes.CDLL(path)
+    P, I, Z = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+    PR = ctypes.POINTER(RouteParams)
+    lib.xshare_workspace_size.argtypes = [I, I, I, I, I, I, PR]
+    lib.xshare_workspace_size.restype = Z
+    lib.xshare_route.argtypes = [P, I, I, I, I, I, PR, P, P, P, P, P, P, P, P, Z, P]
+    lib.xshare_route.restype = I
+    lib.xshare_moe_forward.argtypes = [P, P, P, P, P, I, I, I, I, I, I, I, PR,
+                                       P, P, P, P, P, P, P, Z, P]
+    lib.xshare_moe_forward.restype = I
+    lib.xshare_moe_forward_profiled.argtypes = lib.xshare_moe_forward.argtypes + [P]
+    lib.xshare_moe_forward_profiled.restype = I
+    lib.xshare_stage_name.argtypes = [I]
+    lib.xshare_stage_name.restype = ctypes.c_char_p
+    lib.xshare_strerror.argtypes = [I]
+    lib.xshare_strerror.restype = ctypes.c_char_p
+    return lib
+
+
+LIB = _load()
+
+N_STAGES = 6
+STAGE_NAMES = [LIB.xshare_stage_name(i).decode() for i in range(N_STAGES)]
+
+
+def xshare_strerror(code: int) -> str:
+    return LIB.xshare_strerror(int(code)).decode()
+
+
+def _ptr(t: Optional[torch.Tensor], dtype, name: str, numel: Optional[int] = None) -> Optional[int]:
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if numel is not None and t.numel() < numel:
+        raise ValueError(f"{name} has {t.numel()} elements, needs {numel}")
+    return t.data_ptr()
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _check(rc: int, where: str):
+    if rc != 0:
+        raise XShareError(rc, where)
+
+
+def xshare_workspace_size(B: int, N: int, k: int, d: int, F: int, mode: int,
+                          params: RouteParams) -> int:
+    """Bytes of workspace for these sizes (d = F = 0 for xshare_route); 0 if invalid."""
+    return int(LIB.xshare_workspace_size(B, N, k, d, F, mode, ctypes.byref(params)))
+
+
+def xshare_route(scores: torch.Tensor, k: int, budget: int, mode: int, params: RouteParams,
+                 sel_mask: torch.Tensor, topk_ids: torch.Tensor, topk_w: torch.Tensor,
+                 workspace: torch.Tensor, stats: Optional[torch.Tensor] = None,
+                 expert_counts: Optional[torch.Tensor] = None,
+                 expert_offsets: Optional[torch.Tensor] = None,
+                 perm: Optional[torch.Tensor] = None, stream=None) -> None:
+    """Selection + refinement (+ permutation) on fp32 scores [B, N]; see xshare.h."""
+    B, N = scores.shape
+    rc = LIB.xshare_route(
+        _ptr(scores, torch.float32, "scores"), B, N, k, budget, mode, ctypes.byref(params),
+        _ptr(sel_mask, torch.uint8, "sel_mask", N), _ptr(topk_ids, torch.int32, "topk_ids", B * k),
+        _ptr(topk_w, torch.float32, "topk_w", B * k), _ptr(stats, torch.int32, "stats", STATS_WORDS),
+        _ptr(expert_counts, torch.int32, "expert_counts", N),
+        _ptr(expert_offsets, torch.int32, "expert_offsets", N + 1),
+        _ptr(perm, torch.int32, "perm", B * k),
+        _ptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream))
+    _check(rc, "xshare_route")
+
+
+def xshare_moe_forward(x: torch.Tensor, W_g: torch.Tensor, W_gate: torch.Tensor,
+                       W_up: torch.Tensor, W_down: torch.Tensor, k: int, budget: int, mode: int,
+                       params: RouteParams, y: torch.Tensor, workspace: torch.Tensor,
+                       scores_out: Optional[torch.Tensor] = None,
+                       sel_mask: Optional[torch.Tensor] = None,
+                       topk_ids: Optional[torch.Tensor] = None,
+                       topk_w: Optional[torch.Tensor] = None,
+                       stats: Optional[torch.Tensor] = None, stream=None,
+                       stage_events: Optional[list] = None) -> None:
+    """One MoE-layer forward (routed part) into y [B, d] bf16; see xshare.h.
+
+    With `stage_events` (XS_N_STAGES + 1 torch.cuda.Event objects) the
+    profiled entry point records them between the kernel launches."""
+    B, d = x.shape
+    N = W_g.shape[0]
+    F = W_gate.shape[1]
+    if W_g.shape[1] != d or tuple(W_gate.shape) != (N, F, d) or tuple(W_up.shape) != (N, F, d) \
+            or tuple(W_down.shape) != (N, d, F) or tuple(y.shape) != (B, d):
+        raise ValueError("inconsistent shapes: x [B,d], W_g [N,d], W_gate/W_up [N,F,d], "
+                         "W_down [N,d,F], y [B,d]")
+    args = [
+        _ptr(x, torch.bfloat16, "x"), _ptr(W_g, torch.float32, "W_g"),
+        _ptr(W_gate, torch.bfloat16, "W_gate"), _ptr(W_up, torch.bfloat16, "W_up"),
+        _ptr(W_down, torch.bfloat16, "W_down"), B, d, F, N, k, budget, mode,
+        ctypes.byref(params), _ptr(y, torch.bfloat16, "y"),
+        _ptr(scores_out, torch.float32, "scores_out", B * N),
+        _ptr(sel_mask, torch.uint8, "sel_mask", N), _ptr(topk_ids, torch.int32, "topk_ids", B * k),
+        _ptr(topk_w, torch.float32, "topk_w", B * k), _ptr(stats, torch.int32, "stats", STATS_WORDS),
+        _ptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream)]
+    if stage_events is None:
+        _check(LIB.xshare_moe_forward(*args), "xshare_moe_forward")
+        return
+    if len(stage_events) != N_STAGES + 1:
+        raise ValueError(f"stage_events needs {N_STAGES + 1} events")
+    handles = (ctypes.c_void_p * (N_STAGES + 1))()
+    for i, ev in enumerate(stage_events):
+        if not ev.cuda_event:
+            ev.record()   # torch creates the CUDA event lazily
+        handles[i] = ev.cuda_event
+    _check(LIB.xshare_moe_forward_profiled(*args, handles), "xshare_moe_forward_profiled")
+
+
+def stats_dict(stats: torch.Tensor) -> dict:
+    """Host view of an xs_stats tensor (copies to the host, so it synchronises)."""
+    v = stats.cpu().tolist()
+    return {name: int(v[i]) for i, name in enumerate(STATS_FIELDS)}

@@ -1,0 +1,102 @@
+"""The C-ABI library builds, loads and exports every declared entry point;
+host-side argument checks reject bad calls before anything is launched.
+No compute runs here (no GPU needed)."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "xshare.h")
+
+
+@pytest.fixture(scope="module")
+def X():
+    from paper_2602_07265_gb300 import _build
+    _build.build()
+    from paper_2602_07265_gb300 import xshare
+    return xshare
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(xshare_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    assert declared_functions() == ["xshare_moe_forward", "xshare_moe_forward_profiled",
+                                    "xshare_route", "xshare_stage_name", "xshare_strerror",
+                                    "xshare_workspace_size"]
+
+
+def test_stage_names(X):
+    assert X.STAGE_NAMES == ["router", "select", "gather", "ffn_gate_up", "ffn_down", "combine"]
+    assert X.LIB.xshare_stage_name(6) == b""
+
+
+def test_library_exports_every_declared_symbol(X):
+    from paper_2602_07265_gb300 import _build
+    out = subprocess.run(["nm", "-D", "--defined-only", _build.LIB], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (\w+)$", out, flags=re.M))
+    for name in declared_functions():
+        assert name in exported, name
+        assert getattr(X.LIB, name) is not None
+
+
+def test_strerror_covers_codes(X):
+    for code in (0, -1, -2, -3, -4, -5, -6, -7, 1):
+        s = X.xshare_strerror(code)
+        assert s and "unknown" not in s
+    assert "unknown" in X.xshare_strerror(12345)
+
+
+def _route_rc(X, B=8, N=16, k=4, budget=4, mode=1, prm=None, scores=1 << 20, mask=1 << 20,
+              ids=1 << 20, w=1 << 20, ws=1 << 20, ws_bytes=1 << 20):
+    prm = prm or X.route_params()
+    return X.LIB.xshare_route(scores, B, N, k, budget, mode, ctypes.byref(prm), mask, ids, w,
+                              None, None, None, None, ws, ws_bytes, None)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(B=0), -1), (dict(B=8193), -1), (dict(N=0), -1), (dict(N=1025), -1),
+    (dict(k=0), -1), (dict(k=17), -1), (dict(N=4, k=5), -1),
+    (dict(mode=4), -2), (dict(mode=-1), -2), (dict(budget=-1), -2),
+    (dict(scores=None), -3), (dict(mask=None), -3), (dict(ids=None), -3), (dict(w=None), -3),
+    (dict(scores=(1 << 20) + 4), -5),
+    (dict(ws=None), -4), (dict(ws=(1 << 20) + 16), -4),
+])
+def test_route_rejects_bad_arguments(X, kw, code):
+    assert _route_rc(X, **kw) == code
+
+
+@pytest.mark.parametrize("prm,mode,code", [
+    (dict(k0=-1), 1, -2), (dict(k0=17), 1, -2), (dict(m_r=-1), 3, -2), (dict(m_g=-1), 2, -2),
+    (dict(n_groups=0), 2, -2), (dict(n_groups=3), 2, -2), (dict(n_groups=32), 2, -2),
+    (dict(tokens_per_request=0), 3, -2), (dict(tokens_per_request=3), 3, -2),
+    (dict(tokens_per_request=16), 3, -2),
+])
+def test_route_rejects_bad_params(X, prm, mode, code):
+    assert _route_rc(X, mode=mode, prm=X.route_params(**prm)) == code
+
+
+def test_forward_rejects_bad_shapes(X):
+    prm = X.route_params()
+    P = 1 << 20
+    def rc(d, F, x=P, y=P):
+        return X.LIB.xshare_moe_forward(x, P, P, P, P, 4, d, F, 16, 2, 2, 1, ctypes.byref(prm),
+                                        y, None, None, None, None, None, P, 1 << 20, None)
+    assert rc(100, 256) == -1
+    assert rc(256, 64) == -1
+    assert rc(0, 256) == -1
+    assert rc(256, 256, x=None) == -3
+    assert rc(256, 256, y=P + 8) == -5
+
+
+def test_workspace_size_rejects_invalid(X):
+    prm = X.route_params()
+    assert X.xshare_workspace_size(0, 16, 4, 0, 0, 1, prm) == 0
+    assert X.xshare_workspace_size(8, 16, 4, 100, 256, 1, prm) == 0

@@ -1,0 +1,196 @@
+"""GPU parity of xshare_moe_forward (steps a1-a9) against the oracle, through the C ABI.
+
+Inputs are seeded and synthetic (paper_2602_07265_gb300.workloads); the
+oracle computes everything itself from the same inputs (router in fp64,
+softmax rounded once to fp32, selection on its own fp32 scores, FFN in fp64).
+
+Checks:
+* scores: |p_gpu - p_ref| <= P_RTOL * p_ref elementwise (fp32 router and
+  softmax vs fp64; see P_RTOL);
+* selection: the mask and the top-k ids equal the oracle's, provided the
+  oracle's decision is robust to perturbing its scores by the scores
+  tolerance (checked, never assumed);
+* output: max|y - y_ref| / max|y_ref| <= 2e-2 and ||y - y_ref||_F / ||y_ref||_F
+  <= 1e-2 (bf16 output of an fp32-accumulated path with a bf16 activation).
+At the full DeepSeek-R1 shapes the oracle evaluates sampled tokens only.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import xshare_oracle as O
+from paper_2602_07265_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+# Relative tolerance on the fp32 softmax scores.  h = W_g x is accumulated in
+# fp32 over d terms in a fixed order: each lane adds d/128 float4 steps, then
+# a 5-level butterfly.  With |x_c w_c| ~ 0.02 and partial sums ~ 0.3, the
+# rounding error of h is a few 1e-7 absolute; a softmax score's relative error
+# is at most |dh_j| + |d logsumexp| plus a few ulps of expf and the division.
+P_RTOL = 2e-5
+MAX_REL = 2e-2
+FRO_REL = 1e-2
+
+
+@pytest.fixture(scope="module")
+def X():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2602_07265_gb300 import _build
+    _build.build()
+    from paper_2602_07265_gb300 import xshare
+    return xshare
+
+
+_weights_cache = {}
+
+
+def device_weights(w: W.Workload, seed: int):
+    key = (w.N, w.d, w.F, seed)
+    if key not in _weights_cache:
+        _weights_cache.clear()
+        torch.cuda.empty_cache()
+        _weights_cache[key] = W.expert_weights(w, seed, device="cuda")
+    return _weights_cache[key]
+
+
+def gpu_forward(X, w: W.Workload, x, W_g, weights):
+    dev = torch.device("cuda")
+    Wg, Wu, Wd = weights
+    prm = X.route_params(**w.params())
+    ws = torch.empty(X.xshare_workspace_size(w.B, w.N, w.k, w.d, w.F, w.mode, prm),
+                     dtype=torch.uint8, device=dev)
+    out = dict(
+        y=torch.empty(w.B, w.d, dtype=torch.bfloat16, device=dev),
+        p=torch.empty(w.B, w.N, dtype=torch.float32, device=dev),
+        mask=torch.empty(w.N, dtype=torch.uint8, device=dev),
+        ids=torch.empty(w.B, w.k, dtype=torch.int32, device=dev),
+        w=torch.empty(w.B, w.k, dtype=torch.float32, device=dev),
+        stats=torch.zeros(8, dtype=torch.int32, device=dev),
+    )
+    X.xshare_moe_forward(x.to(dev), W_g.to(dev), Wg, Wu, Wd, w.k, w.budget, w.mode, prm,
+                         out["y"], ws, scores_out=out["p"], sel_mask=out["mask"],
+                         topk_ids=out["ids"], topk_w=out["w"], stats=out["stats"])
+    torch.cuda.synchronize()
+    r = {name: t.cpu() for name, t in out.items()}
+    r["stats"] = X.stats_dict(out["stats"])
+    r["y"] = r["y"].float().numpy().astype(np.float64)
+    for name in ("p", "mask", "ids", "w"):
+        r[name] = r[name].numpy()
+    return r
+
+
+def robust_selection(p, w: W.Workload, rtol: float, trials: int = 4) -> bool:
+    """True if the oracle's routing is unchanged when its scores move by up to rtol."""
+    base = O.route(p, w.k, w.budget, w.mode, **w.params())
+    rng = np.random.default_rng(0)
+    for i in range(trials):
+        f = 1.0 + rtol * (rng.uniform(-1, 1, size=p.shape) if i >= 2 else (1 if i == 0 else -1)
+                          * np.sign(rng.standard_normal(p.shape)))
+        q = (p.astype(np.float64) * f).astype(np.float32)
+        r = O.route(q, w.k, w.budget, w.mode, **w.params())
+        if not (np.array_equal(r["mask"], base["mask"]) and np.array_equal(r["ids"], base["ids"])):
+            return False
+    return True
+
+
+def compare(w, g, x, W_g, weights, tokens=None):
+    Wg, Wu, Wd = weights
+    xb = W.bf16_bits(x)
+
+    def get(e):
+        return W.bf16_bits(Wg[e]), W.bf16_bits(Wu[e]), W.bf16_bits(Wd[e])
+
+    ref = O.moe_forward(xb, W_g.numpy(), get, w.k, w.budget, w.mode, tokens=tokens, **w.params())
+    rel = np.abs(g["p"].astype(np.float64) - ref["p"]) / ref["p"].astype(np.float64)
+    assert rel.max() <= P_RTOL, f"scores: max relative error {rel.max():.3e}"
+    assert robust_selection(ref["p"], w, 2 * P_RTOL), \
+        "oracle decision is within the scores tolerance of a tie: pick another seed"
+    assert np.array_equal(g["mask"], ref["mask"]), "selected set"
+    assert np.array_equal(g["ids"], ref["ids"]), "top-k ids"
+    assert np.allclose(g["w"], ref["w"], rtol=4 * P_RTOL, atol=0), "weights"
+    s = g["stats"]
+    assert s["status"] == 0
+    for key in ("n_selected", "n_used", "union_topk", "max_group_load"):
+        assert s[key] == ref[key], key
+    yg = g["y"] if tokens is None else g["y"][list(tokens)]
+    yr = ref["y"]
+    if np.abs(yr).max() == 0:
+        assert np.all(yg == 0)
+        return ref, 0.0, 0.0
+    max_rel = np.abs(yg - yr).max() / np.abs(yr).max()
+    fro = np.linalg.norm(yg - yr) / np.linalg.norm(yr)
+    assert max_rel <= MAX_REL and fro <= FRO_REL, (max_rel, fro)
+    return ref, max_rel, fro
+
+
+SMALL = [
+    W.TINY, W.TINY.with_(k0=1), W.TINY.with_(mode=W.MODE_TOPK),
+    W.OLMOE.with_(B=8, budget=16), W.OLMOE.with_(B=32, budget=24, k0=1),
+    W.OLMOE.with_(B=64, budget=48), W.OLMOE.with_(B=16, mode=W.MODE_TOPK),
+    W.QWEN3, W.QWEN3.with_(B=16, m_r=5), W.QWEN3.with_(k0=0, budget=16),
+    W.QWEN3.with_(mode=W.MODE_TOPK),
+]
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+@pytest.mark.parametrize("case", range(len(SMALL)))
+def test_forward_parity_small(X, case, seed):
+    w = SMALL[case]
+    x, W_g = W.router_inputs(w, seed)
+    weights = device_weights(w, seed)
+    g = gpu_forward(X, w, x, W_g, weights)
+    compare(w, g, x, W_g, weights)
+
+
+@pytest.mark.parametrize("w", [
+    W.DSR1.with_(B=8), W.DSR1, W.DSR1.with_(B=128, budget=64), W.DSR1.with_(k0=0, budget=32),
+    W.DSR1_GROUP, W.DSR1_GROUP.with_(k0=0, m_g=8),
+], ids=lambda w: f"{w.name}-B{w.B}-m{w.budget}-k0{w.k0}-mg{w.m_g}")
+def test_forward_parity_full_size_sampled(X, w):
+    """DeepSeek-R1-shaped layers at full size; the oracle checks sampled tokens."""
+    x, W_g = W.router_inputs(w, 0)
+    weights = device_weights(w, 0)
+    g = gpu_forward(X, w, x, W_g, weights)
+    tokens = sorted({0, 1, w.B // 2, w.B - 1})
+    compare(w, g, x, W_g, weights, tokens=tokens)
+
+
+@pytest.mark.parametrize("budget,k0", [(0, 0), (3, 0), (0, 1)])
+def test_forward_small_selected_set(X, budget, k0):
+    """|S| = 0 (no routed expert: y = 0), |S| < k, and warm-up only."""
+    w = W.TINY.with_(budget=budget, k0=k0)
+    x, W_g = W.router_inputs(w, 5)
+    weights = device_weights(w, 0)
+    g = gpu_forward(X, w, x, W_g, weights)
+    compare(w, g, x, W_g, weights)
+    if budget == 0 and k0 == 0:
+        assert np.all(g["y"] == 0) and g["stats"]["n_pairs"] == 0
+
+
+def test_forward_single_token(X):
+    w = W.OLMOE.with_(B=1, budget=8, k0=1)
+    x, W_g = W.router_inputs(w, 3)
+    weights = device_weights(w, 3)
+    g = gpu_forward(X, w, x, W_g, weights)
+    compare(w, g, x, W_g, weights)
+
+
+def test_forward_expert_with_many_tokens(X):
+    """Tiles of more than 128 tokens of one expert (popular experts at B = 512)."""
+    w = W.QWEN3.with_(B=512, k0=0, m_r=1, budget=0, tokens_per_request=512)
+    x, W_g = W.router_inputs(w, 1)
+    weights = device_weights(w, 1)
+    g = gpu_forward(X, w, x, W_g, weights)
+    assert max(np.bincount(g["ids"][g["ids"] >= 0])) > 128
+    compare(w, g, x, W_g, weights, tokens=[0, 5, 100, 511])
+
+
+def test_forward_deterministic(X):
+    w = W.OLMOE.with_(B=32, budget=24, k0=1)
+    x, W_g = W.router_inputs(w, 0)
+    weights = device_weights(w, 0)
+    a = gpu_forward(X, w, x, W_g, weights)
+    b = gpu_forward(X, w, x, W_g, weights)
+    assert np.array_equal(a["y"], b["y"]) and np.array_equal(a["p"], b["p"])
