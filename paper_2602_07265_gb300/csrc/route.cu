@@ -80,8 +80,8 @@ __device__ void warp_row_top(const float *__restrict__ prow, int N, int count,
           bi = lane + 32 * q;
         }
     warp_argmax(bv, bi);
-    if (bi == INT_MAX) break;
-    if ((bi & 31) == lane) live &= ~(1u << (bi >> 5));
+    if (bi >= N) bi = -1;  // only with non-finite scores
+    if (bi >= 0 && (bi & 31) == lane) live &= ~(1u << (bi >> 5));
     if (lane == 0) out[r] = bi;
   }
 }
@@ -136,9 +136,11 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
   __syncthreads();
   for (int t = tid; t < B; t += blockDim.x) {
     const int32_t *row = a.toptok + (size_t)t * kMaxK;
-    for (int r = 0; r < k; ++r) s_union[row[r]] = 1;
+    for (int r = 0; r < k; ++r)
+      if ((unsigned)row[r] < (unsigned)N) s_union[row[r]] = 1;
     if (a.mode != XS_MODE_HIER)
-      for (int r = 0; r < a.k0; ++r) s_base[row[r]] = 1;
+      for (int r = 0; r < a.k0; ++r)
+        if ((unsigned)row[r] < (unsigned)N) s_base[row[r]] = 1;
   }
   // ---- a4: batch column scores ----
   for (int j = tid; j < N; j += blockDim.x) s_col[j] = canonical_sum(a.p, N, j, 0, B);
@@ -164,7 +166,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
       for (int x = r0; x < r1; ++x)
         for (int i = 0; i < a.k0; ++i) {
           int e = a.toptok[(size_t)x * kMaxK + i];
-          if ((e & 31) == lane) {
+          if ((unsigned)e < (unsigned)N && (e & 31) == lane) {
             live &= ~(1u << (e >> 5));
             s_base[e] = 1;
           }
@@ -181,7 +183,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
               bi = lane + 32 * q;
             }
         warp_argmax(bv, bi);
-        if (bi == INT_MAX) break;
+        if (bi >= N) break;
         if ((bi & 31) == lane) {
           live &= ~(1u << (bi >> 5));
           s_base[bi] = 1;
@@ -301,7 +303,8 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
             bi = lane + 32 * q;
           }
       warp_argmax(bv, bi);
-      if ((bi & 31) == lane) live &= ~(1u << (bi >> 5));
+      if (bi >= N) bi = -1;  // only with non-finite scores
+      if (bi >= 0 && (bi & 31) == lane) live &= ~(1u << (bi >> 5));
       if (lane == s) {
         my_id = bi;
         my_v = bv;
@@ -321,7 +324,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
   const int P = B * k;
   for (int q = tid; q < P; q += blockDim.x) {
     int e = a.ids[q];
-    if (e >= 0) atomicAdd(&s_counts[e], 1);
+    if ((unsigned)e < (unsigned)N) atomicAdd(&s_counts[e], 1);
   }
   __syncthreads();
   if (warp == 0) {
@@ -390,7 +393,8 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
     const unsigned lt = (1u << lane) - 1u;
     for (int base = 0; base < P; base += 32) {
       const int q = base + lane;
-      const int e = (q < P) ? a.ids[q] : -1;
+      int e = (q < P) ? a.ids[q] : -1;
+      if ((unsigned)e >= (unsigned)N) e = -1;
       const unsigned peers = __match_any_sync(kFull, e);
       const int rank = __popc(peers & lt);
       const int old = (e >= 0) ? s_cursor[e] : 0;
@@ -409,7 +413,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
   }
   if (tid == 0) {
     Meta m;
-    m.n_pairs = B * kp;
+    m.n_pairs = s_off[N];  // == B * kp unless scores were non-finite
     m.n_tiles = s_scal[5];
     m.kprime = kp;
     m.n_selected = nsel;
@@ -425,7 +429,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
       st.n_used = s_scal[4];
       st.union_topk = s_scal[1];
       st.max_group_load = s_scal[2];
-      st.n_pairs = B * kp;
+      st.n_pairs = s_off[N];
       st.status = 0;
       st.reserved[0] = st.reserved[1] = 0;
       *a.stats = st;
@@ -506,6 +510,7 @@ __global__ void __launch_bounds__(256) combine_kernel(const float *__restrict__ 
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
   for (int s = 0; s < kp; ++s) {
     const int r = pos[(size_t)t * k + s];
+    if (r < 0) continue;  // only with non-finite scores
     const float ws = w[(size_t)t * k + s];
     const float4 o = reinterpret_cast<const float4 *>(out + (size_t)r * d)[c4];
     acc.x = fmaf(ws, o.x, acc.x);
