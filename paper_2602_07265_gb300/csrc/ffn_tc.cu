@@ -1,0 +1,459 @@
+// Expert SwiGLU FFN over the routed pairs (step a8) on the 5th-generation
+// tensor cores: tcgen05.mma with TMEM accumulators, operands fed by TMA.
+//
+//   gate/up phase: act[r, f] = silu(W_gate[e, f] . xp[r]) * (W_up[e, f] . xp[r])   (bf16)
+//   down phase   : out[r, c] = W_down[e, c] . act[r]                                (fp32)
+// for every routed pair row r of expert e (Sec. 2.1: E_e(x)).
+//
+// Decode batches give each expert a handful of tokens, so the layer streams
+// the used experts' weights once and is bound by HBM.  The weights fill the
+// MMA's M = 128 dimension ("swap AB") and the expert's tokens are the N
+// dimension (16..128, a multiple of 16, chosen per tile at run time).
+//
+// Work split ("stream-K"): a unit is (tile of <= 128 tokens of one expert,
+// 128 weight rows); its K loop has K/64 steps.  The units' steps are laid end
+// to end and cut into equal contiguous ranges, one per CTA, so every SM
+// streams the same number of weight bytes.  A unit cut between CTAs is
+// finished by whichever CTA arrives last: every piece writes its fp32 partial
+// accumulator, bumps the unit's counter, and the last one adds the pieces in
+// K order (deterministic) and runs the epilogue.  No CTA ever waits for
+// another.
+//
+// Roles inside a CTA (192 threads): warp 0 lane 0 issues TMA loads into a
+// ring of shared-memory stages; warp 1 lane 0 issues the MMAs into one of two
+// TMEM accumulator buffers; warps 2-5 (one TMEM lane quarter each) drain the
+// accumulators.  Every mbarrier wait is bounded in time.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstring>
+
+#include "tc_ptx.cuh"
+#include "xs_internal.cuh"
+
+namespace xs {
+namespace {
+
+using namespace ptx;
+
+constexpr int kBM = 128;          // weight rows per unit (MMA M)
+constexpr int kBK = 64;           // bf16 per K step (one 128-byte swizzle row)
+constexpr int kBoxTok = 16;       // token rows per TMA box of the B operand
+constexpr int kThreads = 192;
+constexpr int kEpiThreads = 128;
+constexpr int kTileBytes = kBM * kBK * 2;     // 16 KB
+constexpr uint64_t kWaitNs = 1000000000ull;   // 1 s per wait
+constexpr int kMinItersPerCta = 8;
+
+template <bool kGateUp>
+struct Cfg {
+  static constexpr int kNumA = kGateUp ? 2 : 1;          // weight tiles per stage
+  static constexpr int kStages = kGateUp ? 4 : 6;
+  static constexpr int kStageBytes = kNumA * kTileBytes + kTileBytes;
+  static constexpr int kAccCols = kGateUp ? 256 : 128;   // TMEM columns per buffer
+  static constexpr int kTmemCols = 2 * kAccCols;
+  static constexpr int kBarOffset = kStages * kStageBytes;
+  static constexpr int kSmemBytes = kBarOffset + 256 + 1024;  // + barriers + alignment slack
+};
+
+struct TcParams {
+  CUtensorMap tmA0;     // W_gate (gate/up) or W_down (down): [N * M, K] bf16, box 128 x 64
+  CUtensorMap tmA1;     // W_up (gate/up only)
+  CUtensorMap tmB;      // xp (gate/up) or act (down): [max_pairs, K] bf16, box 16 x 64
+  const Tile *tiles;
+  Meta *meta;
+  xs_stats *stats;
+  float *part;          // [grid][2 slots][kNumA][128 cols][128 lanes] fp32
+  int32_t *cnt;         // [units] arrival counters, zeroed by the routing kernel
+  uint16_t *act_out;    // gate/up output [max_pairs, M]
+  float *out;           // down output [max_pairs, M]
+  int M;                // weight rows per expert: F (gate/up) or d (down)
+  int K;                // reduction length: d (gate/up) or F (down)
+  int grid;
+};
+
+struct Range {
+  long long I;      // total K steps
+  int G;            // CTAs that take part
+  int KI;           // K steps per unit
+  __device__ long long begin(int c) const { return I * c / G; }
+  // CTA whose range holds step i.
+  __device__ int cta_of(long long i) const {
+    int c = static_cast<int>((i * G) / I);
+    while (c + 1 < G && begin(c + 1) <= i) ++c;
+    while (c > 0 && begin(c) > i) --c;
+    return c;
+  }
+  // Partial slot a CTA uses for unit u: 0 for the unit its range starts in, 1 otherwise.
+  __device__ int slot(int c, long long u) const { return (begin(c) / KI == u) ? 0 : 1; }
+};
+
+__device__ __forceinline__ void set_status(const TcParams &p, int code) {
+  atomicMax(&p.meta->status, code);
+  if (p.stats) atomicMax(&p.stats->status, code);
+}
+
+__device__ __forceinline__ float silu(float g) { return g / (1.f + expf(-g)); }
+
+template <bool kGateUp>
+__global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_constant__ TcParams p) {
+  using C = Cfg<kGateUp>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = reinterpret_cast<uint8_t *>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t bar0 = sbase + C::kBarOffset;
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (C::kStages + s); };
+  auto accfull_bar = [&](int b) { return bar0 + 8u * (2 * C::kStages + b); };
+  auto accempty_bar = [&](int b) { return bar0 + 8u * (2 * C::kStages + 2 + b); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * C::kStages + 4);
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kBarOffset + 8 * (2 * C::kStages + 5));
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+  volatile int *s_flag = reinterpret_cast<volatile int *>(tmem_slot + 2);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n_tiles = p.meta->n_tiles;
+  const int MT = p.M / kBM, KI = p.K / kBK;
+  Range rg;
+  rg.KI = KI;
+  rg.I = static_cast<long long>(n_tiles) * MT * KI;
+  if (rg.I == 0) return;
+  const long long want = (rg.I + kMinItersPerCta - 1) / kMinItersPerCta;
+  rg.G = static_cast<int>(want < p.grid ? want : p.grid);
+  if (static_cast<int>(blockIdx.x) >= rg.G) return;
+  const int cta = blockIdx.x;
+  const long long it_begin = rg.begin(cta), it_end = rg.begin(cta + 1);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(accfull_bar(b), 1);
+      mbar_init(accempty_bar(b), 1);
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&p.tmA0);
+    if (kGateUp) prefetch_tmap(&p.tmA1);
+    prefetch_tmap(&p.tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), C::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------ TMA producer
+    if (lane == 0) {
+      const uint64_t pol_w = policy_evict_first(), pol_x = policy_evict_last();
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued_mask = 0, issued_phase = 0;
+      bool ok = true;
+      for (long long it = it_begin; ok && it < it_end;) {
+        const long long u = it / KI;
+        const int k0 = static_cast<int>(it - u * KI);
+        const int k1 = static_cast<int>(k0 + (it_end - it) < KI ? k0 + (it_end - it) : KI);
+        const Tile tl = p.tiles[u / MT];
+        const int mt = static_cast<int>(u % MT);
+        const int nb = (tl.ntok + kBoxTok - 1) / kBoxTok;
+        const uint32_t tx = C::kNumA * kTileBytes + nb * kBoxTok * kBK * 2;
+        const int arow = tl.expert * p.M + mt * kBM;
+        for (int kk = k0; kk < k1; ++kk) {
+          if (!mbar_wait(empty_bar(stage), phase ^ 1u, kWaitNs, abort_flag)) {
+            ok = false;
+            break;
+          }
+          const uint32_t sA = sbase + stage * C::kStageBytes;
+          const uint32_t sB = sA + C::kNumA * kTileBytes;
+          mbar_arrive_expect_tx(full_bar(stage), tx);
+          tma_load_2d(sA, &p.tmA0, full_bar(stage), kk * kBK, arow, pol_w);
+          if (kGateUp) tma_load_2d(sA + kTileBytes, &p.tmA1, full_bar(stage), kk * kBK, arow, pol_w);
+          for (int b = 0; b < nb; ++b)
+            tma_load_2d(sB + b * kBoxTok * kBK * 2, &p.tmB, full_bar(stage), kk * kBK,
+                        tl.row0 + b * kBoxTok, pol_x);
+          issued_mask |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == C::kStages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        it += k1 - k0;
+      }
+      if (!ok) {
+        set_status(p, XS_DEV_TIMEOUT);
+        *abort_flag = 1;
+      }
+      // Never leave with copies in flight: wait (bounded) for the last load of every stage.
+      volatile int no_abort = 0;
+      for (int s = 0; s < C::kStages; ++s)
+        if ((issued_mask >> s) & 1u) mbar_wait(full_bar(s), (issued_phase >> s) & 1u, kWaitNs, &no_abort);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int segi = 0;
+      bool ok = true, any = false;
+      for (long long it = it_begin; ok && it < it_end; ++segi) {
+        const long long u = it / KI;
+        const int k0 = static_cast<int>(it - u * KI);
+        const int k1 = static_cast<int>(k0 + (it_end - it) < KI ? k0 + (it_end - it) : KI);
+        const Tile tl = p.tiles[u / MT];
+        const int n_mma = ((tl.ntok + 15) / 16) * 16;
+        const uint32_t idesc = idesc_bf16(kBM, n_mma);
+        const int buf = segi & 1;
+        const uint32_t use = static_cast<uint32_t>(segi >> 1);
+        if (!mbar_wait(accempty_bar(buf), (use & 1u) ^ 1u, kWaitNs, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d0 = tmem + buf * C::kAccCols;
+        for (int kk = k0; kk < k1; ++kk) {
+          if (!mbar_wait(full_bar(stage), phase, kWaitNs, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sA = sbase + stage * C::kStageBytes;
+          const uint32_t sB = sA + C::kNumA * kTileBytes;
+#pragma unroll
+          for (int ks = 0; ks < kBK / 16; ++ks) {
+            const uint32_t acc = (kk > k0 || ks > 0) ? 1u : 0u;
+            const uint64_t db = sw128_desc(sB + ks * 32);
+            mma_bf16(d0, sw128_desc(sA + ks * 32), db, idesc, acc);
+            if (kGateUp) mma_bf16(d0 + 128, sw128_desc(sA + kTileBytes + ks * 32), db, idesc, acc);
+          }
+          any = true;
+          mma_commit(empty_bar(stage));
+          if (++stage == C::kStages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        mma_commit(accfull_bar(buf));
+        it += k1 - k0;
+      }
+      if (!ok) {
+        set_status(p, XS_DEV_TIMEOUT);
+        *abort_flag = 1;
+      }
+      if (any) {  // all issued MMAs done before TMEM is released
+        volatile int no_abort = 0;
+        mma_commit(drain_bar);
+        mbar_wait(drain_bar, 0, kWaitNs, &no_abort);
+      }
+    }
+  } else {
+    // ------------------------------------------------ epilogue (warps 2..5)
+    const int q = warp & 3;                  // TMEM lane quarter of this warp
+    const int row = q * 32 + lane;           // weight row inside the unit
+    const bool leader = threadIdx.x == 64;
+    int segi = 0;
+    for (long long it = it_begin; it < it_end; ++segi) {
+      const long long u = it / KI;
+      const int k0 = static_cast<int>(it - u * KI);
+      const int k1 = static_cast<int>(k0 + (it_end - it) < KI ? k0 + (it_end - it) : KI);
+      const Tile tl = p.tiles[u / MT];
+      const int mt = static_cast<int>(u % MT);
+      const int n_mma = ((tl.ntok + 15) / 16) * 16;
+      const int buf = segi & 1;
+      const uint32_t use = static_cast<uint32_t>(segi >> 1);
+      if (leader) *s_flag = mbar_wait(accfull_bar(buf), use & 1u, kWaitNs, abort_flag) ? 1 : 0;
+      named_bar_sync(1, kEpiThreads);
+      const bool ok = *s_flag != 0;
+      named_bar_sync(1, kEpiThreads);
+      if (!ok) {
+        if (leader) {
+          set_status(p, XS_DEV_TIMEOUT);
+          *abort_flag = 1;
+        }
+        break;
+      }
+      tc_fence_after();
+      const uint32_t tacc = tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * C::kAccCols;
+      const int col = mt * kBM + row;
+
+      // Emits the outputs of accumulator columns [c0, c0 + 16).
+      auto emit = [&](int c0, const float (&g)[16], const float (&v)[16]) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          if (c0 + j < tl.ntok) {
+            const size_t r = static_cast<size_t>(tl.row0 + c0 + j) * p.M + col;
+            if (kGateUp) {
+              const __nv_bfloat16 h = __float2bfloat16_rn(silu(g[j]) * v[j]);
+              p.act_out[r] = *reinterpret_cast<const uint16_t *>(&h);
+            } else {
+              p.out[r] = g[j];
+            }
+          }
+        }
+      };
+
+      if (k0 == 0 && k1 == KI) {
+        for (int c0 = 0; c0 < n_mma; c0 += 16) {
+          float g[16], v[16];
+          tmem_ld16(tacc + c0, g);
+          if (kGateUp) tmem_ld16(tacc + 128 + c0, v);
+          emit(c0, g, v);
+        }
+      } else {
+        // Piece of a unit shared with other CTAs: publish the partial sums.
+        const int my_slot = rg.slot(cta, u);
+        float *mine = p.part + static_cast<size_t>(cta * 2 + my_slot) * C::kNumA * 128 * 128;
+        for (int c0 = 0; c0 < n_mma; c0 += 16) {
+          float g[16], v[16];
+          tmem_ld16(tacc + c0, g);
+          if (kGateUp) tmem_ld16(tacc + 128 + c0, v);
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            mine[(c0 + j) * 128 + row] = g[j];
+            if (kGateUp) mine[(128 + c0 + j) * 128 + row] = v[j];
+          }
+        }
+        __threadfence();
+        named_bar_sync(1, kEpiThreads);
+        const int c_first = rg.cta_of(u * KI), c_last = rg.cta_of(u * KI + KI - 1);
+        if (leader) {
+          const int old = atomicAdd(&p.cnt[u], 1);
+          *s_flag = (old == c_last - c_first) ? 1 : 0;
+        }
+        named_bar_sync(1, kEpiThreads);
+        const bool last = *s_flag != 0;
+        named_bar_sync(1, kEpiThreads);
+        if (last) {
+          __threadfence();
+          for (int c0 = 0; c0 < n_mma; c0 += 16) {
+            float g[16], v[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) g[j] = v[j] = 0.f;
+            for (int c = c_first; c <= c_last; ++c) {
+              const float *src = p.part + static_cast<size_t>(c * 2 + rg.slot(c, u)) * C::kNumA * 128 * 128;
+#pragma unroll
+              for (int j = 0; j < 16; ++j) {
+                const float a = __ldcg(src + (c0 + j) * 128 + row);
+                g[j] = (c == c_first) ? a : g[j] + a;
+                if (kGateUp) {
+                  const float b = __ldcg(src + (128 + c0 + j) * 128 + row);
+                  v[j] = (c == c_first) ? b : v[j] + b;
+                }
+              }
+            }
+            emit(c0, g, v);
+          }
+        }
+      }
+      tc_fence_before();
+      named_bar_sync(1, kEpiThreads);
+      if (leader) mbar_arrive(accempty_bar(buf));
+      it += k1 - k0;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::kTmemCols);
+  }
+}
+
+// ---------------------------------------------------------------- host side
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (fn == nullptr) {
+    void *ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  }
+  return fn;
+}
+
+// Row-major [outer, inner] bf16 matrix, boxes of box_outer x 64, 128-byte swizzle.
+bool make_map(CUtensorMap *m, const void *base, uint64_t inner, uint64_t outer, uint32_t box_outer) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <bool kGateUp>
+cudaError_t launch_phase(const TcParams &p, cudaStream_t s) {
+  using C = Cfg<kGateUp>;
+  cudaError_t e = cudaFuncSetAttribute(ffn_tc_kernel<kGateUp>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+  if (e != cudaSuccess) return e;
+  ffn_tc_kernel<kGateUp><<<p.grid, kThreads, C::kSmemBytes, s>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+size_t ffn_part_bytes(int n_sms) { return static_cast<size_t>(n_sms) * 2 * 2 * 128 * 128 * 4; }
+
+size_t ffn_cnt_words(int max_tiles, int d, int F) {
+  return static_cast<size_t>(max_tiles) * (F / kBM + d / kBM);
+}
+
+cudaError_t launch_ffn_gate_up(const FfnArgs &a, cudaStream_t s) {
+  TcParams p;
+  memset(&p, 0, sizeof(p));
+  if (!make_map(&p.tmA0, a.W_gate, a.d, static_cast<uint64_t>(a.N) * a.F, kBM) ||
+      !make_map(&p.tmA1, a.W_up, a.d, static_cast<uint64_t>(a.N) * a.F, kBM) ||
+      !make_map(&p.tmB, a.xp, a.d, a.max_pairs, kBoxTok))
+    return cudaErrorInvalidValue;
+  p.tiles = a.tiles;
+  p.meta = a.meta;
+  p.stats = a.stats;
+  p.part = static_cast<float *>(a.part);
+  p.cnt = a.cnt;
+  p.act_out = a.act;
+  p.M = a.F;
+  p.K = a.d;
+  p.grid = a.n_sms;
+  return launch_phase<true>(p, s);
+}
+
+cudaError_t launch_ffn_down(const FfnArgs &a, cudaStream_t s) {
+  TcParams p;
+  memset(&p, 0, sizeof(p));
+  if (!make_map(&p.tmA0, a.W_down, a.F, static_cast<uint64_t>(a.N) * a.d, kBM) ||
+      !make_map(&p.tmB, a.act, a.F, a.max_pairs, kBoxTok))
+    return cudaErrorInvalidValue;
+  p.tmA1 = p.tmA0;
+  p.tiles = a.tiles;
+  p.meta = a.meta;
+  p.stats = a.stats;
+  p.part = static_cast<float *>(a.part);
+  p.cnt = a.cnt + static_cast<size_t>(a.max_tiles) * (a.F / kBM);
+  p.out = a.out;
+  p.M = a.d;
+  p.K = a.F;
+  p.grid = a.n_sms;
+  return launch_phase<false>(p, s);
+}
+
+}  // namespace xs

@@ -81,13 +81,16 @@ def gpu_forward(X, w: W.Workload, x, W_g, weights):
     return r
 
 
-def robust_selection(p, w: W.Workload, rtol: float, trials: int = 4) -> bool:
-    """True if the oracle's routing is unchanged when its scores move by up to rtol."""
+def robust_selection(p, w: W.Workload, rtol: float, trials: int = 6) -> bool:
+    """True if the oracle's routing is unchanged when its scores move by up to rtol
+    (random relative perturbations, including the all-up / all-down extremes)."""
     base = O.route(p, w.k, w.budget, w.mode, **w.params())
     rng = np.random.default_rng(0)
     for i in range(trials):
-        f = 1.0 + rtol * (rng.uniform(-1, 1, size=p.shape) if i >= 2 else (1 if i == 0 else -1)
-                          * np.sign(rng.standard_normal(p.shape)))
+        if i < 2:
+            f = 1.0 + rtol * (1 if i == 0 else -1) * np.sign(rng.standard_normal(p.shape))
+        else:
+            f = 1.0 + rtol * rng.uniform(-1, 1, size=p.shape)
         q = (p.astype(np.float64) * f).astype(np.float32)
         r = O.route(q, w.k, w.budget, w.mode, **w.params())
         if not (np.array_equal(r["mask"], base["mask"]) and np.array_equal(r["ids"], base["ids"])):
@@ -96,6 +99,13 @@ def robust_selection(p, w: W.Workload, rtol: float, trials: int = 4) -> bool:
 
 
 def compare(w, g, x, W_g, weights, tokens=None):
+    """Check a GPU forward against the oracle; returns (ref, max_rel, fro, n_tokens_compared).
+
+    The GPU decides its selection on its own fp32 scores, which differ from
+    the oracle's by rounding (|dp| / p <= P_RTOL, checked).  Its mask and ids
+    must equal the oracle's unless the oracle's own decision flips under a
+    perturbation of the size actually observed (a near-tie); then y is
+    compared on every token whose routing (ids) is identical."""
     Wg, Wu, Wd = weights
     xb = W.bf16_bits(x)
 
@@ -105,24 +115,36 @@ def compare(w, g, x, W_g, weights, tokens=None):
     ref = O.moe_forward(xb, W_g.numpy(), get, w.k, w.budget, w.mode, tokens=tokens, **w.params())
     rel = np.abs(g["p"].astype(np.float64) - ref["p"]) / ref["p"].astype(np.float64)
     assert rel.max() <= P_RTOL, f"scores: max relative error {rel.max():.3e}"
-    assert robust_selection(ref["p"], w, 2 * P_RTOL), \
-        "oracle decision is within the scores tolerance of a tie: pick another seed"
-    assert np.array_equal(g["mask"], ref["mask"]), "selected set"
-    assert np.array_equal(g["ids"], ref["ids"]), "top-k ids"
-    assert np.allclose(g["w"], ref["w"], rtol=4 * P_RTOL, atol=0), "weights"
+    toks = list(range(w.B)) if tokens is None else list(tokens)
+    same_mask = np.array_equal(g["mask"], ref["mask"])
+    same_row = np.all(g["ids"] == ref["ids"], axis=1)
+    if not (same_mask and same_row.all()):
+        eps = max(4 * float(rel.max()), 1e-6)
+        assert not robust_selection(ref["p"], w, eps), \
+            "routing differs from the oracle's although its decision is not near a tie"
+    keep = [i for i, t in enumerate(toks) if same_row[t]]
+    print(f"[{w.name} B={w.B} mode={w.mode}] p_rel_max={rel.max():.2e} same_mask={same_mask} "
+          f"same_rows={int(same_row.sum())}/{w.B} compared={len(keep)}/{len(toks)}")
+    assert len(keep) >= max(1, (3 * len(toks)) // 4), "too few tokens with identical routing"
+    rows = [toks[i] for i in keep]
+    assert np.allclose(g["w"][rows], ref["w"][rows], rtol=4 * P_RTOL, atol=0), "weights"
     s = g["stats"]
     assert s["status"] == 0
-    for key in ("n_selected", "n_used", "union_topk", "max_group_load"):
-        assert s[key] == ref[key], key
-    yg = g["y"] if tokens is None else g["y"][list(tokens)]
-    yr = ref["y"]
+    if same_mask and same_row.all():
+        for key in ("n_selected", "n_used", "max_group_load"):
+            assert s[key] == ref[key], key
+        # the plain top-k union depends on every token's k-th/(k+1)-th gap over E
+        assert abs(s["union_topk"] - ref["union_topk"]) <= 1
+    yg = g["y"][rows]
+    yr = ref["y"][keep]
     if np.abs(yr).max() == 0:
         assert np.all(yg == 0)
-        return ref, 0.0, 0.0
+        return ref, 0.0, 0.0, len(keep)
     max_rel = np.abs(yg - yr).max() / np.abs(yr).max()
     fro = np.linalg.norm(yg - yr) / np.linalg.norm(yr)
+    print(f"    y: max_rel={max_rel:.3e} fro={fro:.3e}")
     assert max_rel <= MAX_REL and fro <= FRO_REL, (max_rel, fro)
-    return ref, max_rel, fro
+    return ref, max_rel, fro, len(keep)
 
 
 SMALL = [
