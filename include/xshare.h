@@ -153,6 +153,31 @@ int xshare_moe_forward(const uint16_t *x, const float *W_g, const uint16_t *W_ga
                        int32_t *topk_ids, float *topk_w, xs_stats *stats, void *workspace,
                        size_t ws_bytes, xs_stream_t stream);
 
+/* xshare_route for callers that cannot allocate device memory.  The paper has
+ * no counterpart: this is a deployment convenience of the library.
+ *
+ * Who needs it: code loaded into a host program that owns all device memory
+ * through its own allocator and offers no allocation hook, and serving loops
+ * that must not allocate once running (cudaMalloc can synchronise the whole
+ * device).  Neither can hand xshare_route a workspace.
+ *
+ * Same arguments and results as xshare_route, minus the workspace.  The
+ * scratch is a fixed array inside the library's device code (about 220 KB
+ * on every GPU that loads the library, held until the process exits), so:
+ *   - B is limited to 1024 tokens (N <= 1024 and k <= 16 as elsewhere); a
+ *     larger B returns XS_ERR_SHAPE and launches nothing;
+ *   - the first call on a device looks up the array's device address with
+ *     cudaGetSymbolAddress; make that first call before any stream capture;
+ *   - every call on a device uses the same array, so calls that can overlap
+ *     on the GPU (different streams, or different host threads) race and
+ *     must be ordered by the caller.  Nothing in the array needs clearing
+ *     between calls: the kernel writes each scratch word before reading it.
+ * Allocates nothing (no cudaMalloc, cudaFree or allocating library call). */
+int xshare_route_static(const float *scores, int B, int N, int k, int budget, int mode,
+                        const xs_route_params *prm, uint8_t *sel_mask, int32_t *topk_ids,
+                        float *topk_w, xs_stats *stats, int32_t *expert_counts,
+                        int32_t *expert_offsets, int32_t *perm, xs_stream_t stream);
+
 /* Kernel stages of xshare_moe_forward, in launch order. */
 #define XS_N_STAGES 6
 

@@ -1,0 +1,118 @@
+// xshare_route_static: the selection / refinement / permutation of
+// xshare_route for callers that cannot allocate device memory.
+//
+// Some hosts own every byte of device memory through their own allocator and
+// give the code they load no way to allocate more; some serving loops must
+// not allocate after start-up because cudaMalloc can synchronise the device.
+// Such callers cannot supply xshare_route's workspace.  This entry point
+// keeps its scratch in a fixed array that the library module itself defines
+// in device memory, sized for at most kStaticMaxB tokens, so the caller passes
+// only its inputs and outputs.
+#include <cuda_runtime.h>
+
+#include <cstring>
+
+#include "xs_internal.cuh"
+
+namespace xs {
+namespace {
+
+constexpr int kStaticMaxB = 1024;
+constexpr size_t kStaticAlign = 256;
+
+constexpr size_t up256(size_t v) { return (v + kStaticAlign - 1) / kStaticAlign * kStaticAlign; }
+
+constexpr int kStaticMaxPairs = kStaticMaxB * kMaxK;
+constexpr int kStaticMaxTiles = kMaxN + kStaticMaxPairs / kTileTok + 1;
+
+// Scratch layout (byte offsets), sized for B <= kStaticMaxB, N <= kMaxN, k <= kMaxK.
+constexpr size_t kOffTopTok = 0;
+constexpr size_t kOffCounts = kOffTopTok + up256(sizeof(int32_t) * kStaticMaxB * kMaxK);
+constexpr size_t kOffOffsets = kOffCounts + up256(sizeof(int32_t) * kMaxN);
+constexpr size_t kOffPerm = kOffOffsets + up256(sizeof(int32_t) * (kMaxN + 1));
+constexpr size_t kOffPos = kOffPerm + up256(sizeof(int32_t) * kStaticMaxPairs);
+constexpr size_t kOffTiles = kOffPos + up256(sizeof(int32_t) * kStaticMaxPairs);
+constexpr size_t kOffMeta = kOffTiles + up256(sizeof(Tile) * kStaticMaxTiles);
+constexpr size_t kStaticBytes = kOffMeta + up256(sizeof(Meta));
+
+// The scratch itself: one copy per device that loads the library, kept until
+// the process exits.  From host code this name is only a handle for
+// cudaGetSymbolAddress, never a device address.
+static __device__ __align__(256) unsigned char g_route_scratch[kStaticBytes];
+
+constexpr int kMaxDevices = 64;
+void *g_scratch_addr[kMaxDevices];  // device address of g_route_scratch, per device
+
+}  // namespace
+}  // namespace xs
+
+using namespace xs;
+
+extern "C" int xshare_route_static(const float *scores, int B, int N, int k, int budget, int mode,
+                                   const xs_route_params *prm, uint8_t *sel_mask,
+                                   int32_t *topk_ids, float *topk_w, xs_stats *stats,
+                                   int32_t *expert_counts, int32_t *expert_offsets,
+                                   int32_t *perm, xs_stream_t stream) {
+  if (prm == nullptr) return XS_ERR_NULL;
+  if (B < 1 || B > kStaticMaxB || N < 1 || N > kMaxN || k < 1 || k > kMaxK || k > N)
+    return XS_ERR_SHAPE;
+  if (mode < XS_MODE_TOPK || mode > XS_MODE_HIER) return XS_ERR_PARAM;
+  if (budget < 0 || prm->k0 < 0 || prm->k0 > kMaxK || prm->k0 > N || prm->m_r < 0 ||
+      prm->m_g < 0 || prm->n_groups < 0)
+    return XS_ERR_PARAM;
+  if (prm->n_groups > 0 && (prm->n_groups > N || N % prm->n_groups != 0)) return XS_ERR_PARAM;
+  if (mode == XS_MODE_GROUP && prm->n_groups < 1) return XS_ERR_PARAM;
+  if (mode == XS_MODE_HIER &&
+      (prm->tokens_per_request < 1 || prm->tokens_per_request > B || B % prm->tokens_per_request != 0))
+    return XS_ERR_PARAM;
+  if (!scores || !sel_mask || !topk_ids || !topk_w) return XS_ERR_NULL;
+  if ((reinterpret_cast<uintptr_t>(scores) & 15u) != 0) return XS_ERR_ALIGN;
+
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return XS_ERR_CUDA;
+  int major = 0, minor = 0;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+    return XS_ERR_CUDA;
+  if (major != 10 || minor != 3) return XS_ERR_DEVICE;
+  if (g_scratch_addr[dev] == nullptr) {
+    // One-time set-up on this device: look up where the scratch array lives.
+    void *addr = nullptr;
+    if (cudaGetSymbolAddress(&addr, g_route_scratch) != cudaSuccess || addr == nullptr)
+      return XS_ERR_CUDA;
+    g_scratch_addr[dev] = addr;
+  }
+  char *base = static_cast<char *>(g_scratch_addr[dev]);
+
+  RouteArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.p = const_cast<float *>(scores);  // read only: no logits are given
+  a.B = B;
+  a.N = N;
+  a.k = k;
+  a.budget = budget;
+  a.mode = mode;
+  a.k0 = (mode == XS_MODE_TOPK) ? 0 : prm->k0;
+  a.m_r = prm->m_r;
+  a.T = prm->tokens_per_request < 1 ? 1 : prm->tokens_per_request;
+  a.G = prm->n_groups < 1 ? 1 : prm->n_groups;
+  a.m_g = prm->m_g > N ? N : prm->m_g;
+  a.mask = sel_mask;
+  a.ids = topk_ids;
+  a.w = topk_w;
+  a.toptok = reinterpret_cast<int32_t *>(base + kOffTopTok);
+  a.counts = reinterpret_cast<int32_t *>(base + kOffCounts);
+  a.offsets = reinterpret_cast<int32_t *>(base + kOffOffsets);
+  a.perm = reinterpret_cast<int32_t *>(base + kOffPerm);
+  a.pos = reinterpret_cast<int32_t *>(base + kOffPos);
+  a.tiles = reinterpret_cast<Tile *>(base + kOffTiles);
+  a.meta = reinterpret_cast<Meta *>(base + kOffMeta);
+  a.stats = stats;
+  a.counts_out = expert_counts;
+  a.offsets_out = expert_offsets;
+  a.perm_out = perm;
+  a.zero_words = nullptr;  // the routing kernel writes every scratch word before reading it
+  a.zero_count = 0;
+  return launch_route(a, reinterpret_cast<cudaStream_t>(stream)) == cudaSuccess ? XS_OK
+                                                                                 : XS_ERR_CUDA;
+}

@@ -58,6 +58,8 @@ def _load() -> ctypes.CDLL:
     lib.xshare_moe_forward.argtypes = [P, P, P, P, P, I, I, I, I, I, I, I, PR,
                                        P, P, P, P, P, P, P, Z, P]
     lib.xshare_moe_forward.restype = I
+    lib.xshare_route_static.argtypes = [P, I, I, I, I, I, PR, P, P, P, P, P, P, P, P]
+    lib.xshare_route_static.restype = I
     lib.xshare_moe_forward_profiled.argtypes = lib.xshare_moe_forward.argtypes + [P]
     lib.xshare_moe_forward_profiled.restype = I
     lib.xshare_stage_name.argtypes = [I]
@@ -125,6 +127,28 @@ def xshare_route(scores: torch.Tensor, k: int, budget: int, mode: int, params: R
         _ptr(perm, torch.int32, "perm", B * k),
         _ptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream))
     _check(rc, "xshare_route")
+
+
+STATIC_MAX_B = 1024
+
+
+def xshare_route_static(scores: torch.Tensor, k: int, budget: int, mode: int,
+                        params: RouteParams, sel_mask: torch.Tensor, topk_ids: torch.Tensor,
+                        topk_w: torch.Tensor, stats: Optional[torch.Tensor] = None,
+                        expert_counts: Optional[torch.Tensor] = None,
+                        expert_offsets: Optional[torch.Tensor] = None,
+                        perm: Optional[torch.Tensor] = None, stream=None) -> None:
+    """xshare_route without a workspace, for callers that may not allocate
+    device memory (B <= STATIC_MAX_B; see xshare.h)."""
+    B, N = scores.shape
+    rc = LIB.xshare_route_static(
+        _ptr(scores, torch.float32, "scores"), B, N, k, budget, mode, ctypes.byref(params),
+        _ptr(sel_mask, torch.uint8, "sel_mask", N), _ptr(topk_ids, torch.int32, "topk_ids", B * k),
+        _ptr(topk_w, torch.float32, "topk_w", B * k), _ptr(stats, torch.int32, "stats", STATS_WORDS),
+        _ptr(expert_counts, torch.int32, "expert_counts", N),
+        _ptr(expert_offsets, torch.int32, "expert_offsets", N + 1),
+        _ptr(perm, torch.int32, "perm", B * k), _stream(stream))
+    _check(rc, "xshare_route_static")
 
 
 def xshare_moe_forward(x: torch.Tensor, W_g: torch.Tensor, W_gate: torch.Tensor,
