@@ -56,19 +56,12 @@ __device__ __forceinline__ float canonical_sum(const float *__restrict__ p, int 
   return acc;
 }
 
-// One warp ranks the experts of row `t` of p: writes the `count` best of E,
-// best first, to out[0..count).  kMaxQ = columns held per lane (N <= 32 kMaxQ).
-template <int kMaxQ>
-__device__ void warp_row_top(const float *__restrict__ prow, int N, int count,
-                             int32_t *__restrict__ out, int lane) {
-  float vals[kMaxQ];
-  unsigned live = 0;
-#pragma unroll
-  for (int q = 0; q < kMaxQ; ++q) {
-    int j = lane + 32 * q;
-    vals[q] = (j < N) ? prow[j] : -INFINITY;
-    if (j < N) live |= 1u << q;
-  }
+// Ranks the values a warp holds (lane l holds columns l + 32 q, q < kMaxQ,
+// valid where bit q of `live` is set) and returns, best first, up to
+// `count` expert ids through `emit(r, id)`; -1 ends the list early.
+template <int kMaxQ, class Emit>
+__device__ __forceinline__ void warp_rank(const float (&vals)[kMaxQ], unsigned live, int count,
+                                          int N, int lane, Emit emit) {
   for (int r = 0; r < count; ++r) {
     float bv = -INFINITY;
     int bi = INT_MAX;
@@ -80,14 +73,26 @@ __device__ void warp_row_top(const float *__restrict__ prow, int N, int count,
           bi = lane + 32 * q;
         }
     warp_argmax(bv, bi);
-    if (bi >= N) bi = -1;  // only with non-finite scores
-    if (bi >= 0 && (bi & 31) == lane) live &= ~(1u << (bi >> 5));
-    if (lane == 0) out[r] = bi;
+    if (bi >= N) return;  // fewer candidates than `count`
+    if ((bi & 31) == lane) live &= ~(1u << (bi >> 5));
+    emit(r, bi, bv);
   }
 }
 
+// The whole selection in one CTA (steps a2-a7):
+//   1. per token (one warp each): dense softmax of the logits (or the given
+//      scores) held in registers, then its ranked top-max(k, k0) over E, which
+//      marks the plain top-k union and the warm-up set S_0;
+//   2. canonical column sums (one thread per expert) and, for HIER, the
+//      per-request selections of Algorithm 3 (one warp per request);
+//   3. the budgeted selection (rank counting in shared memory);
+//   4. per token the top-k' inside S with renormalised weights, counting the
+//      pairs per expert on the way;
+//   5. prefix sums, FFN tiles, and the stable scatter of the pairs.
+// The score matrix and the ids are staged in shared memory when they fit.
 template <int kMaxQ>
 __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
+  extern __shared__ float dsm[];
   __shared__ uint8_t s_mask[kMaxN];   // S
   __shared__ uint8_t s_base[kMaxN];   // S_0 (or the union of the S_r for HIER)
   __shared__ uint8_t s_union[kMaxN];  // union of plain top-k
@@ -95,30 +100,17 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
   __shared__ int32_t s_counts[kMaxN];
   __shared__ int32_t s_off[kMaxN + 1];
   __shared__ int32_t s_toff[kMaxN + 1];
-  __shared__ int32_t s_cursor[kMaxN];
   __shared__ int32_t s_avail[kMaxN];
-  __shared__ int32_t s_scal[8];      // 0:|S| 1:union 2:maxload 3:R* 4:|U| 5:tiles 6:|S_0|
+  __shared__ int32_t s_scal[8];      // 3:R* 4:|U| 5:tiles
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nwarps = blockDim.x >> 5;
   const int B = a.B, N = a.N, k = a.k;
   const int kk = max(k, a.k0);  // ranked list length per token
+  float *ps = a.p_smem ? dsm : nullptr;
+  int32_t *ids_s = a.ids_smem ? reinterpret_cast<int32_t *>(dsm + (a.p_smem ? B * N : 0)) : nullptr;
+  const float *P = ps ? ps : a.p;
 
-  // ---- a2: dense softmax over all N experts (if logits are given) ----
-  if (a.logits != nullptr) {
-    for (int t = warp; t < B; t += nwarps) {
-      const float *h = a.logits + (size_t)t * N;
-      float mx = -INFINITY;
-      for (int j = lane; j < N; j += 32) mx = fmaxf(mx, h[j]);
-#pragma unroll
-      for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, o));
-      float sum = 0.f;
-      for (int j = lane; j < N; j += 32) sum = __fadd_rn(sum, expf(h[j] - mx));
-#pragma unroll
-      for (int o = 16; o; o >>= 1) sum = __fadd_rn(sum, __shfl_xor_sync(kFull, sum, o));
-      for (int j = lane; j < N; j += 32) a.p[(size_t)t * N + j] = __fdiv_rn(expf(h[j] - mx), sum);
-    }
-  }
   for (int j = tid; j < N; j += blockDim.x) {
     s_mask[j] = 0;
     s_base[j] = 0;
@@ -130,23 +122,70 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
     for (int i = tid; i < a.zero_count; i += blockDim.x) a.zero_words[i] = 0;
   __syncthreads();
 
-  // ---- a3: per-token ranked top-kk over E (warm-up and plain top-k union) ----
-  for (int t = warp; t < B; t += nwarps)
-    warp_row_top<kMaxQ>(a.p + (size_t)t * N, N, kk, a.toptok + (size_t)t * kMaxK, lane);
-  __syncthreads();
-  for (int t = tid; t < B; t += blockDim.x) {
-    const int32_t *row = a.toptok + (size_t)t * kMaxK;
-    for (int r = 0; r < k; ++r)
-      if ((unsigned)row[r] < (unsigned)N) s_union[row[r]] = 1;
-    if (a.mode != XS_MODE_HIER)
-      for (int r = 0; r < a.k0; ++r)
-        if ((unsigned)row[r] < (unsigned)N) s_base[row[r]] = 1;
+  // ---- 1. scores (a2) and per-token ranking over E (a3) ----
+  for (int t = warp; t < B; t += nwarps) {
+    float vals[kMaxQ];
+    unsigned live = 0;
+    if (a.logits != nullptr) {
+      const float *hrow = a.logits + (size_t)t * N;
+      float mx = -INFINITY;
+#pragma unroll
+      for (int q = 0; q < kMaxQ; ++q) {
+        const int j = lane + 32 * q;
+        vals[q] = (j < N) ? hrow[j] : -INFINITY;
+        mx = fmaxf(mx, vals[q]);
+      }
+#pragma unroll
+      for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, o));
+      float sum = 0.f;
+#pragma unroll
+      for (int q = 0; q < kMaxQ; ++q) {
+        vals[q] = (lane + 32 * q < N) ? expf(vals[q] - mx) : 0.f;
+        sum = __fadd_rn(sum, vals[q]);
+      }
+#pragma unroll
+      for (int o = 16; o; o >>= 1) sum = __fadd_rn(sum, __shfl_xor_sync(kFull, sum, o));
+#pragma unroll
+      for (int q = 0; q < kMaxQ; ++q) {
+        const int j = lane + 32 * q;
+        if (j < N) {
+          vals[q] = __fdiv_rn(vals[q], sum);
+          a.p[(size_t)t * N + j] = vals[q];
+          if (ps) ps[t * N + j] = vals[q];
+          live |= 1u << q;
+        }
+      }
+    } else {
+#pragma unroll
+      for (int q = 0; q < kMaxQ; ++q) {
+        const int j = lane + 32 * q;
+        vals[q] = (j < N) ? a.p[(size_t)t * N + j] : -INFINITY;
+        if (j < N) {
+          if (ps) ps[t * N + j] = vals[q];
+          live |= 1u << q;
+        }
+      }
+    }
+    const bool hier = a.mode == XS_MODE_HIER;
+    int32_t *top = a.toptok + (size_t)t * kMaxK;
+    warp_rank<kMaxQ>(vals, live, kk, N, lane, [&](int r, int id, float) {
+      if (lane == 0) {
+        if (r < k) s_union[id] = 1;
+        if (r < a.k0) {
+          if (hier)
+            top[r] = id;
+          else
+            s_base[id] = 1;
+        }
+      }
+    });
   }
-  // ---- a4: batch column scores ----
-  for (int j = tid; j < N; j += blockDim.x) s_col[j] = canonical_sum(a.p, N, j, 0, B);
   __syncthreads();
 
-  // ---- a5': HIER per-request selection (Algorithm 3), one warp per request ----
+  // ---- 2. batch column scores (a4) ----
+  for (int j = tid; j < N; j += blockDim.x) s_col[j] = canonical_sum(P, N, j, 0, B);
+
+  // ---- 2'. HIER: per-request selection (Algorithm 3), one warp per request ----
   if (a.mode == XS_MODE_HIER) {
     const int T = a.T, R = B / T;
     for (int r = warp; r < R; r += nwarps) {
@@ -155,51 +194,36 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
       unsigned live = 0;
 #pragma unroll
       for (int q = 0; q < kMaxQ; ++q) {
-        int j = lane + 32 * q;
+        const int j = lane + 32 * q;
         sc[q] = 0.f;
         if (j < N) {
-          sc[q] = canonical_sum(a.p, N, j, r0, r1);
+          sc[q] = canonical_sum(P, N, j, r0, r1);
           live |= 1u << q;
         }
       }
       // S0_r: union of Top k0 over the request's tokens.
       for (int x = r0; x < r1; ++x)
         for (int i = 0; i < a.k0; ++i) {
-          int e = a.toptok[(size_t)x * kMaxK + i];
+          const int e = a.toptok[(size_t)x * kMaxK + i];
           if ((unsigned)e < (unsigned)N && (e & 31) == lane) {
             live &= ~(1u << (e >> 5));
             s_base[e] = 1;
           }
         }
       // S_r = S0_r + Top m_r(scores_r, E \ S0_r).
-      for (int c = 0; c < a.m_r; ++c) {
-        float bv = -INFINITY;
-        int bi = INT_MAX;
-#pragma unroll
-        for (int q = 0; q < kMaxQ; ++q)
-          if ((live >> q) & 1u)
-            if (better(sc[q], lane + 32 * q, bv, bi)) {
-              bv = sc[q];
-              bi = lane + 32 * q;
-            }
-        warp_argmax(bv, bi);
-        if (bi >= N) break;
-        if ((bi & 31) == lane) {
-          live &= ~(1u << (bi >> 5));
-          s_base[bi] = 1;
-        }
-      }
+      warp_rank<kMaxQ>(sc, live, a.m_r, N, lane, [&](int, int id, float) {
+        if (lane == 0) s_base[id] = 1;
+      });
     }
-    __syncthreads();
   }
+  __syncthreads();
 
-  // ---- a5: budgeted selection ----
-  for (int j = tid; j < N; j += blockDim.x)
-    if (s_base[j]) atomicAdd(&s_scal[6], 1);
+  // ---- 3. budgeted selection (a5) ----
   if (a.mode == XS_MODE_GROUP) {
+    const int size = N / a.G;
+    const int n_base = __syncthreads_count(tid < N && s_base[tid]);
     for (int j = tid; j < N; j += blockDim.x) s_avail[j] = 0;
     __syncthreads();
-    const int size = N / a.G;
     for (int j = tid; j < N; j += blockDim.x)
       if (!s_base[j]) atomicAdd(&s_avail[j / size], 1);
     __syncthreads();
@@ -208,10 +232,10 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
       // min(R, avail_g).  R* is the first round count reaching m_g * G.
       int maxav = 0;
       for (int g = 0; g < a.G; ++g) maxav = max(maxav, s_avail[g]);
-      long long target = (long long)a.m_g * a.G;
+      const long long target = (long long)a.m_g * a.G;
       int R = 0;
       for (;;) {
-        long long tot = s_scal[6];
+        long long tot = n_base;
         for (int g = 0; g < a.G; ++g) tot += min(R, s_avail[g]);
         if (tot >= target || R >= maxav) break;
         ++R;
@@ -251,88 +275,69 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
   __syncthreads();
 
   // ---- statistics ----
-  {
+  const int nsel = __syncthreads_count(tid < N && s_mask[tid]);
+  const int n_union = __syncthreads_count(tid < N && s_union[tid]);
+  if (warp == 0) {
     const int G = a.G >= 1 ? a.G : 1;
     const int size = N / G;
-    for (int j = tid; j < N; j += blockDim.x) {
-      if (s_mask[j]) atomicAdd(&s_scal[0], 1);
-      if (s_union[j]) atomicAdd(&s_scal[1], 1);
+    int best = 0;
+    for (int g = lane; g < G; g += 32) {
+      int c = 0;
+      for (int j = g * size; j < (g + 1) * size; ++j) c += s_mask[j];
+      best = max(best, c);
     }
-    if (warp == 0) {
-      int best = 0;
-      for (int g = lane; g < G; g += 32) {
-        int c = 0;
-        for (int j = g * size; j < (g + 1) * size; ++j) c += s_mask[j];
-        best = max(best, c);
-      }
 #pragma unroll
-      for (int o = 16; o; o >>= 1) best = max(best, __shfl_xor_sync(kFull, best, o));
-      if (lane == 0) s_scal[2] = best;
-    }
+    for (int o = 16; o; o >>= 1) best = max(best, __shfl_xor_sync(kFull, best, o));
+    if (lane == 0) s_scal[2] = best;
   }
   for (int j = tid; j < N; j += blockDim.x) a.mask[j] = s_mask[j];
-  __syncthreads();
-  const int nsel = s_scal[0];
   const int kp = min(k, nsel);
 
-  // ---- a6: refinement, Top k'(G_i, S) with renormalised weights ----
+  // ---- 4. refinement (a6): Top k'(G_i, S), renormalised weights, pair counts ----
   for (int t = warp; t < B; t += nwarps) {
-    const float *prow = a.p + (size_t)t * N;
     float vals[kMaxQ];
     unsigned live = 0;
 #pragma unroll
     for (int q = 0; q < kMaxQ; ++q) {
-      int j = lane + 32 * q;
+      const int j = lane + 32 * q;
       vals[q] = 0.f;
       if (j < N && s_mask[j]) {
-        vals[q] = prow[j];
+        vals[q] = P[(size_t)t * N + j];
         live |= 1u << q;
       }
     }
-    int my_id = -1;      // lane s keeps slot s
+    int my_id = -1;  // lane s keeps slot s
     float my_v = 0.f;
     float D = 0.f;
-    for (int s = 0; s < kp; ++s) {
-      float bv = -INFINITY;
-      int bi = INT_MAX;
-#pragma unroll
-      for (int q = 0; q < kMaxQ; ++q)
-        if ((live >> q) & 1u)
-          if (better(vals[q], lane + 32 * q, bv, bi)) {
-            bv = vals[q];
-            bi = lane + 32 * q;
-          }
-      warp_argmax(bv, bi);
-      if (bi >= N) bi = -1;  // only with non-finite scores
-      if (bi >= 0 && (bi & 31) == lane) live &= ~(1u << (bi >> 5));
-      if (lane == s) {
-        my_id = bi;
-        my_v = bv;
+    int got = 0;
+    warp_rank<kMaxQ>(vals, live, kp, N, lane, [&](int r, int id, float v) {
+      if (lane == r) {
+        my_id = id;
+        my_v = v;
       }
-      D = __fadd_rn(D, bv);  // slot order, identical on every lane
-    }
+      D = __fadd_rn(D, v);  // slot order, identical on every lane
+      got = r + 1;
+    });
     if (lane < k) {
       float wv = 0.f;
-      if (lane < kp) wv = (D > 0.f) ? __fdiv_rn(my_v, D) : __fdiv_rn(1.f, (float)kp);
-      a.ids[(size_t)t * k + lane] = (lane < kp) ? my_id : -1;
+      if (lane < got) wv = (D > 0.f) ? __fdiv_rn(my_v, D) : __fdiv_rn(1.f, (float)got);
+      const int id = (lane < got) ? my_id : -1;
+      a.ids[(size_t)t * k + lane] = id;
       a.w[(size_t)t * k + lane] = wv;
+      if (ids_s) ids_s[t * k + lane] = id;
+      if (id >= 0) atomicAdd(&s_counts[id], 1);
     }
   }
   __syncthreads();
 
-  // ---- a7: permutation (counting sort by expert, stable in (token, slot)) ----
-  const int P = B * k;
-  for (int q = tid; q < P; q += blockDim.x) {
-    int e = a.ids[q];
-    if ((unsigned)e < (unsigned)N) atomicAdd(&s_counts[e], 1);
-  }
-  __syncthreads();
+  // ---- 5. permutation (a7): counting sort by expert, stable in (token, slot) ----
+  const int P2 = B * k;
   if (warp == 0) {
-    // Exclusive scans over N (<= 1024) of counts and of tile counts, 32 per lane.
+    // Exclusive scans over N (<= 1024) of counts and of tile counts, per/lane each.
     const int per = (N + 31) / 32;
     int c_sum = 0, t_sum = 0, used = 0;
     for (int i = 0; i < per; ++i) {
-      int e = lane * per + i;
+      const int e = lane * per + i;
       if (e < N) {
         c_sum += s_counts[e];
         t_sum += (s_counts[e] + kTileTok - 1) / kTileTok;
@@ -342,8 +347,8 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
     int c_inc = c_sum, t_inc = t_sum, u_inc = used;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      int c2 = __shfl_up_sync(kFull, c_inc, o), t2 = __shfl_up_sync(kFull, t_inc, o);
-      int u2 = __shfl_up_sync(kFull, u_inc, o);
+      const int c2 = __shfl_up_sync(kFull, c_inc, o), t2 = __shfl_up_sync(kFull, t_inc, o);
+      const int u2 = __shfl_up_sync(kFull, u_inc, o);
       if (lane >= o) {
         c_inc += c2;
         t_inc += t2;
@@ -352,7 +357,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
     }
     int c_run = c_inc - c_sum, t_run = t_inc - t_sum;
     for (int i = 0; i < per; ++i) {
-      int e = lane * per + i;
+      const int e = lane * per + i;
       if (e < N) {
         s_off[e] = c_run;
         s_toff[e] = t_run;
@@ -370,7 +375,6 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
   __syncthreads();
   for (int e = tid; e < N; e += blockDim.x) {
     const int c = s_counts[e];
-    s_cursor[e] = s_off[e];
     a.counts[e] = c;
     a.offsets[e] = s_off[e];
     if (a.counts_out) a.counts_out[e] = c;
@@ -390,97 +394,132 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
   }
   __syncthreads();
   if (warp == 0) {
+    // s_counts becomes the running cursor of each expert (warp 0 only from here).
+    for (int e = lane; e < N; e += 32) s_counts[e] = s_off[e];
+    __syncwarp();
     const unsigned lt = (1u << lane) - 1u;
-    for (int base = 0; base < P; base += 32) {
+    const int32_t *ids = ids_s ? ids_s : a.ids;
+    for (int base = 0; base < P2; base += 32) {
       const int q = base + lane;
-      int e = (q < P) ? a.ids[q] : -1;
+      int e = (q < P2) ? ids[q] : -1;
       if ((unsigned)e >= (unsigned)N) e = -1;
       const unsigned peers = __match_any_sync(kFull, e);
       const int rank = __popc(peers & lt);
-      const int old = (e >= 0) ? s_cursor[e] : 0;
+      const int old = (e >= 0) ? s_counts[e] : 0;
       __syncwarp();
       if (e >= 0) {
         const int r = old + rank;
         a.perm[r] = q;
         a.pos[q] = r;
         if (a.perm_out) a.perm_out[r] = q;
-        if (rank == 0) s_cursor[e] = old + __popc(peers);
-      } else if (q < P) {
+        if (rank == 0) s_counts[e] = old + __popc(peers);
+      } else if (q < P2) {
         a.pos[q] = -1;
       }
       __syncwarp();
     }
-  }
-  if (tid == 0) {
-    Meta m;
-    m.n_pairs = s_off[N];  // == B * kp unless scores were non-finite
-    m.n_tiles = s_scal[5];
-    m.kprime = kp;
-    m.n_selected = nsel;
-    m.n_used = s_scal[4];
-    m.union_topk = s_scal[1];
-    m.max_group_load = s_scal[2];
-    m.status = 0;
-    for (int i = 0; i < 8; ++i) m.pad[i] = 0;
-    *a.meta = m;
-    if (a.stats) {
-      xs_stats st;
-      st.n_selected = nsel;
-      st.n_used = s_scal[4];
-      st.union_topk = s_scal[1];
-      st.max_group_load = s_scal[2];
-      st.n_pairs = s_off[N];
-      st.status = 0;
-      st.reserved[0] = st.reserved[1] = 0;
-      *a.stats = st;
+    if (lane == 0) {
+      Meta m;
+      m.n_pairs = s_off[N];  // == B * kp unless scores were non-finite
+      m.n_tiles = s_scal[5];
+      m.kprime = kp;
+      m.n_selected = nsel;
+      m.n_used = s_scal[4];
+      m.union_topk = n_union;
+      m.max_group_load = s_scal[2];
+      m.status = 0;
+      for (int i = 0; i < 8; ++i) m.pad[i] = 0;
+      *a.meta = m;
+      if (a.stats) {
+        xs_stats st;
+        st.n_selected = nsel;
+        st.n_used = s_scal[4];
+        st.union_topk = n_union;
+        st.max_group_load = s_scal[2];
+        st.n_pairs = s_off[N];
+        st.status = 0;
+        st.reserved[0] = st.reserved[1] = 0;
+        *a.stats = st;
+      }
     }
   }
 }
 
-// ---- a1: router logits h = W_g x, fp32.  Block = 8 experts x 8 tokens; warp
-// w owns expert e0 + w; a lane sums its slice of d (float4 steps), then the
-// warp adds the 32 lane sums with a butterfly.
+// ---- a1: router logits h = W_g x, fp32.
+// A block owns 8 tokens x 8 experts; its 8 warps split the d dimension into 8
+// contiguous slices.  A lane walks its slice in float4 steps and keeps the
+// 8 x 8 outer-product sums in registers (each W_g and x value loaded once per
+// block, 16 loads per 256 FMAs).  A butterfly reduce-scatter over the 32
+// lanes leaves each lane two finished sums, and the 8 warp partials are
+// added in warp order through shared memory: a fixed order, so h is
+// reproducible bit for bit.
 constexpr int kRtTok = 8;
 constexpr int kRtExp = 8;
+constexpr int kRtWarps = 8;
+constexpr int kRtOut = kRtTok * kRtExp;   // 64 sums per lane before the reduction
 
-__global__ void __launch_bounds__(256) router_logits_kernel(const uint16_t *__restrict__ x,
-                                                            const float *__restrict__ Wg,
-                                                            float *__restrict__ h, int B,
-                                                            int N, int d) {
+__global__ void __launch_bounds__(kRtWarps * 32) router_logits_kernel(
+    const uint16_t *__restrict__ x, const float *__restrict__ Wg, float *__restrict__ h, int B,
+    int N, int d) {
+  __shared__ float red[kRtWarps][kRtOut];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int e = blockIdx.x * kRtExp + warp;
-  const int t0 = blockIdx.y * kRtTok;
-  float acc[kRtTok];
+  const int e0 = blockIdx.x * kRtExp, t0 = blockIdx.y * kRtTok;
+  const int d4 = d / 4;
+  const int c_begin = warp * (d4 / kRtWarps), c_end = (warp + 1) * (d4 / kRtWarps);
+  float acc[kRtOut];
 #pragma unroll
-  for (int j = 0; j < kRtTok; ++j) acc[j] = 0.f;
-  if (e < N) {
-    const float4 *wrow = reinterpret_cast<const float4 *>(Wg + (size_t)e * d);
-    for (int c4 = lane; c4 < d / 4; c4 += 32) {
-      const float4 wv = __ldg(wrow + c4);
+  for (int i = 0; i < kRtOut; ++i) acc[i] = 0.f;
+  const float4 *wbase = reinterpret_cast<const float4 *>(Wg);
+  const uint2 *xbase = reinterpret_cast<const uint2 *>(x);
+#pragma unroll 1
+  for (int c4 = c_begin + lane; c4 < c_end; c4 += 32) {
+    float xf[kRtTok][4];
+#pragma unroll
+    for (int j = 0; j < kRtTok; ++j) {
+      uint2 v = make_uint2(0u, 0u);
+      if (t0 + j < B) v = __ldg(xbase + (size_t)(t0 + j) * d4 + c4);
+      xf[j][0] = __uint_as_float(v.x << 16);
+      xf[j][1] = __uint_as_float(v.x & 0xffff0000u);
+      xf[j][2] = __uint_as_float(v.y << 16);
+      xf[j][3] = __uint_as_float(v.y & 0xffff0000u);
+    }
+#pragma unroll
+    for (int e = 0; e < kRtExp; ++e) {
+      float4 wv = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (e0 + e < N) wv = __ldg(wbase + (size_t)(e0 + e) * d4 + c4);
 #pragma unroll
       for (int j = 0; j < kRtTok; ++j) {
-        if (t0 + j < B) {
-          const uint2 xv = __ldg(reinterpret_cast<const uint2 *>(x + (size_t)(t0 + j) * d) + c4);
-          const float x0 = __uint_as_float(xv.x << 16), x1 = __uint_as_float(xv.x & 0xffff0000u);
-          const float x2 = __uint_as_float(xv.y << 16), x3 = __uint_as_float(xv.y & 0xffff0000u);
-          acc[j] = fmaf(x0, wv.x, acc[j]);
-          acc[j] = fmaf(x1, wv.y, acc[j]);
-          acc[j] = fmaf(x2, wv.z, acc[j]);
-          acc[j] = fmaf(x3, wv.w, acc[j]);
-        }
+        float a = acc[j * kRtExp + e];
+        a = fmaf(xf[j][0], wv.x, a);
+        a = fmaf(xf[j][1], wv.y, a);
+        a = fmaf(xf[j][2], wv.z, a);
+        a = fmaf(xf[j][3], wv.w, a);
+        acc[j * kRtExp + e] = a;
       }
     }
   }
+  // Reduce-scatter: after the step with offset o a lane keeps the half of its
+  // values selected by bit o of its lane id; after five steps lane l holds
+  // the complete sums of outputs 2l and 2l + 1.
 #pragma unroll
-  for (int j = 0; j < kRtTok; ++j)
+  for (int o = 16, n = kRtOut / 2; o >= 1; o >>= 1, n >>= 1) {
+    const bool upper = (lane & o) != 0;
 #pragma unroll
-    for (int o = 16; o; o >>= 1) acc[j] += __shfl_xor_sync(kFull, acc[j], o);
-  if (e < N) {
-    float mine = 0.f;
+    for (int i = 0; i < n; ++i) {
+      const float lo = acc[i], hi = acc[i + n];
+      const float recv = __shfl_xor_sync(kFull, upper ? lo : hi, o);
+      acc[i] = (upper ? hi : lo) + recv;
+    }
+  }
+  red[warp][2 * lane] = acc[0];
+  red[warp][2 * lane + 1] = acc[1];
+  __syncthreads();
+  if (threadIdx.x < kRtOut) {
+    float s = red[0][threadIdx.x];
 #pragma unroll
-    for (int j = 0; j < kRtTok; ++j)
-      if (lane == j) mine = acc[j];
-    if (lane < kRtTok && t0 + lane < B) h[(size_t)(t0 + lane) * N + e] = mine;
+    for (int w = 1; w < kRtWarps; ++w) s += red[w][threadIdx.x];
+    const int t = t0 + threadIdx.x / kRtExp, e = e0 + threadIdx.x % kRtExp;
+    if (t < B && e < N) h[(size_t)t * N + e] = s;
   }
 }
 
@@ -528,22 +567,37 @@ __global__ void __launch_bounds__(256) combine_kernel(const float *__restrict__ 
 
 }  // namespace
 
-cudaError_t launch_route(const RouteArgs &a, cudaStream_t s) {
-  if (a.N <= 64)
-    route_kernel<2><<<1, kRouteThreads, 0, s>>>(a);
-  else if (a.N <= 128)
-    route_kernel<4><<<1, kRouteThreads, 0, s>>>(a);
-  else if (a.N <= 256)
-    route_kernel<8><<<1, kRouteThreads, 0, s>>>(a);
-  else
-    route_kernel<32><<<1, kRouteThreads, 0, s>>>(a);
+size_t route_dynamic_smem(int B, int N, int k, bool *p_smem, bool *ids_smem) {
+  const size_t p_bytes = (size_t)B * N * 4, ids_bytes = (size_t)B * k * 4;
+  *p_smem = p_bytes <= kRouteSmemP;
+  *ids_smem = ids_bytes <= kRouteSmemIds;
+  return (*p_smem ? p_bytes : 0) + (*ids_smem ? ids_bytes : 0);
+}
+
+template <int kMaxQ>
+cudaError_t launch_route_q(RouteArgs a, cudaStream_t s) {
+  bool ps = false, is = false;
+  const size_t dyn = route_dynamic_smem(a.B, a.N, a.k, &ps, &is);
+  a.p_smem = ps ? 1 : 0;
+  a.ids_smem = is ? 1 : 0;
+  cudaError_t e = cudaFuncSetAttribute(route_kernel<kMaxQ>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+  if (e != cudaSuccess) return e;
+  route_kernel<kMaxQ><<<1, kRouteThreads, dyn, s>>>(a);
   return cudaGetLastError();
+}
+
+cudaError_t launch_route(const RouteArgs &a, cudaStream_t s) {
+  if (a.N <= 64) return launch_route_q<2>(a, s);
+  if (a.N <= 128) return launch_route_q<4>(a, s);
+  if (a.N <= 256) return launch_route_q<8>(a, s);
+  return launch_route_q<32>(a, s);
 }
 
 cudaError_t launch_router_logits(const uint16_t *x, const float *Wg, float *h, int B, int N,
                                  int d, cudaStream_t s) {
   dim3 grid((N + kRtExp - 1) / kRtExp, (B + kRtTok - 1) / kRtTok);
-  router_logits_kernel<<<grid, 256, 0, s>>>(x, Wg, h, B, N, d);
+  router_logits_kernel<<<grid, kRtWarps * 32, 0, s>>>(x, Wg, h, B, N, d);
   return cudaGetLastError();
 }
 

@@ -14,6 +14,8 @@ constexpr int kMaxK = 16;       // top-k and warm-up k0
 constexpr int kMaxB = 8192;     // tokens
 constexpr int kTileTok = 128;   // tokens of one expert handled by one FFN tile
 constexpr int kRouteThreads = 1024;
+constexpr size_t kRouteSmemP = 128 * 1024;   // score matrix staged in shared memory up to this size
+constexpr size_t kRouteSmemIds = 64 * 1024;  // top-k ids staged in shared memory up to this size
 
 // One FFN work tile: up to kTileTok consecutive rows of the permuted pair
 // list, all routed to `expert`.
@@ -68,6 +70,8 @@ struct RouteArgs {
   int32_t *perm_out;
   int32_t *zero_words;   // nullable: region cleared for the FFN kernels
   int zero_count;
+  int p_smem;            // set by launch_route: scores staged in shared memory
+  int ids_smem;          // set by launch_route: ids staged in shared memory
 };
 
 cudaError_t launch_route(const RouteArgs &a, cudaStream_t s);
