@@ -14,8 +14,9 @@ constexpr int kMaxK = 16;       // top-k and warm-up k0
 constexpr int kMaxB = 8192;     // tokens
 constexpr int kTileTok = 128;   // tokens of one expert handled by one FFN tile
 constexpr int kRouteThreads = 1024;
-constexpr size_t kRouteSmemP = 128 * 1024;   // score matrix staged in shared memory up to this size
+constexpr size_t kRouteSmemP = 96 * 1024;    // score matrix staged in shared memory up to this size
 constexpr size_t kRouteSmemIds = 64 * 1024;  // top-k ids staged in shared memory up to this size
+constexpr int kScatterMaxN = 256;            // parallel stable scatter up to this many experts
 
 // One FFN work tile: up to kTileTok consecutive rows of the permuted pair
 // list, all routed to `expert`.
