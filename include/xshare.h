@@ -178,7 +178,9 @@ int xshare_route_static(const float *scores, int B, int N, int k, int budget, in
                         float *topk_w, xs_stats *stats, int32_t *expert_counts,
                         int32_t *expert_offsets, int32_t *perm, xs_stream_t stream);
 
-/* Kernel stages of xshare_moe_forward, in launch order. */
+/* Kernel stages of xshare_moe_forward, in launch order: router logits,
+ * selection (softmax, Algorithms 2-6, refinement, permutation), token
+ * gather, SwiGLU gate/up, SwiGLU down, weighted combine. */
 #define XS_N_STAGES 6
 
 /* xshare_moe_forward that also records CUDA events on `stream` between its

@@ -126,7 +126,7 @@ Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms) {
     pl.act = take((size_t)pl.max_pairs * F * 2);
     pl.out = take((size_t)pl.max_pairs * d * 4);
     pl.ffn_part = take(ffn_part_bytes(n_sms));
-    pl.ffn_cnt = take(ffn_cnt_words(pl.max_tiles, d, F) * 4);
+    pl.ffn_cnt = take(ffn_cnt_words(pl.max_tiles, B, d, F) * 4);
   }
   pl.total = o;
   return pl;
@@ -208,7 +208,7 @@ int forward_impl(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
   if (topk_w) a.w = topk_w;
   a.stats = stats;
   a.zero_words = at<int32_t>(workspace, pl.ffn_cnt);
-  a.zero_count = (int)ffn_cnt_words(pl.max_tiles, d, F);
+  a.zero_count = (int)ffn_cnt_words(pl.max_tiles, B, d, F);
 
   FfnArgs f;
   std::memset(&f, 0, sizeof(f));

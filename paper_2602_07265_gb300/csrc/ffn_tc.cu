@@ -114,6 +114,8 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
   volatile int *s_flag = reinterpret_cast<volatile int *>(tmem_slot + 2);
 
+  pdl_wait();
+  pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n_tiles = p.meta->n_tiles;
   const int MT = p.M / kBM, KI = p.K / kBK;
@@ -406,15 +408,15 @@ cudaError_t launch_phase(const TcParams &p, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(ffn_tc_kernel<kGateUp>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
   if (e != cudaSuccess) return e;
-  ffn_tc_kernel<kGateUp><<<p.grid, kThreads, C::kSmemBytes, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(ffn_tc_kernel<kGateUp>, dim3(p.grid), dim3(kThreads), C::kSmemBytes, s, p);
 }
 
 }  // namespace
 
 size_t ffn_part_bytes(int n_sms) { return static_cast<size_t>(n_sms) * 2 * 2 * 128 * 128 * 4; }
 
-size_t ffn_cnt_words(int max_tiles, int d, int F) {
+size_t ffn_cnt_words(int max_tiles, int B, int d, int F) {
+  (void)B;
   return static_cast<size_t>(max_tiles) * (F / kBM + d / kBM);
 }
 

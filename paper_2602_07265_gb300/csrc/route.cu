@@ -196,6 +196,8 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
   __shared__ int32_t s_tmp[200];
   __shared__ int32_t s_scal[8];       // 0:R* 1:max group load 2:|U| 3:tiles 4:pairs
 
+  pdl_wait();
+  pdl_trigger();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nwarps = blockDim.x >> 5;
   const int B = a.B, N = a.N, k = a.k;
@@ -560,6 +562,8 @@ __global__ void __launch_bounds__(kRtWarps * 32) router_logits_kernel(
     const uint16_t *__restrict__ x, const float *__restrict__ Wg, float *__restrict__ h, int B,
     int N, int d) {
   __shared__ float red[kRtWarps][kRtOut];
+  pdl_wait();
+  pdl_trigger();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int e0 = blockIdx.x * kRtExp, t0 = blockIdx.y * kRtTok;
   const int d4 = d / 4;
@@ -629,6 +633,8 @@ __global__ void __launch_bounds__(256) gather_kernel(const uint16_t *__restrict_
                                                      const int32_t *__restrict__ perm,
                                                      const Meta *__restrict__ meta,
                                                      uint16_t *__restrict__ xp, int d, int k) {
+  pdl_wait();
+  pdl_trigger();
   const int row = blockIdx.x;
   if (row >= meta->n_pairs) return;
   const int t = perm[row] / k;
@@ -643,6 +649,8 @@ __global__ void __launch_bounds__(256) combine_kernel(const float *__restrict__ 
                                                       const float *__restrict__ w,
                                                       const Meta *__restrict__ meta,
                                                       uint16_t *__restrict__ y, int d, int k) {
+  pdl_wait();
+  pdl_trigger();
   const int t = blockIdx.y;
   const int c4 = blockIdx.x * blockDim.x + threadIdx.x;
   if (c4 >= d / 4) return;
@@ -685,8 +693,7 @@ cudaError_t launch_route_q(RouteArgs a, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(route_kernel<kMaxQ>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
   if (e != cudaSuccess) return e;
-  route_kernel<kMaxQ><<<1, kRouteThreads, dyn, s>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(route_kernel<kMaxQ>, dim3(1), dim3(kRouteThreads), dyn, s, a);
 }
 
 cudaError_t launch_route(const RouteArgs &a, cudaStream_t s) {
@@ -699,22 +706,19 @@ cudaError_t launch_route(const RouteArgs &a, cudaStream_t s) {
 cudaError_t launch_router_logits(const uint16_t *x, const float *Wg, float *h, int B, int N,
                                  int d, cudaStream_t s) {
   dim3 grid((N + kRtExp - 1) / kRtExp, (B + kRtTok - 1) / kRtTok);
-  router_logits_kernel<<<grid, kRtWarps * 32, 0, s>>>(x, Wg, h, B, N, d);
-  return cudaGetLastError();
+  return launch_pdl(router_logits_kernel, grid, dim3(kRtWarps * 32), 0, s, x, Wg, h, B, N, d);
 }
 
 cudaError_t launch_gather(const uint16_t *x, const int32_t *perm, const Meta *meta,
                           uint16_t *xp, int max_pairs, int d, int k, cudaStream_t s) {
-  gather_kernel<<<max_pairs, 256, 0, s>>>(x, perm, meta, xp, d, k);
-  return cudaGetLastError();
+  return launch_pdl(gather_kernel, dim3(max_pairs), dim3(256), 0, s, x, perm, meta, xp, d, k);
 }
 
 cudaError_t launch_combine(const float *out, const int32_t *pos, const float *w,
                            const Meta *meta, uint16_t *y, int B, int d, int k,
                            cudaStream_t s) {
   dim3 grid((d / 4 + 255) / 256, B);
-  combine_kernel<<<grid, 256, 0, s>>>(out, pos, w, meta, y, d, k);
-  return cudaGetLastError();
+  return launch_pdl(combine_kernel, grid, dim3(256), 0, s, out, pos, w, meta, y, d, k);
 }
 
 }  // namespace xs

@@ -4,10 +4,39 @@
 #include <cuda_runtime.h>
 #include <cstddef>
 #include <cstdint>
+#include <utility>
 
 #include "xshare.h"
 
 namespace xs {
+
+// Programmatic dependent launch.  Every kernel of the library is launched
+// with programmatic stream serialization and starts with pdl_wait(), which
+// returns once all work before it in the stream has completed and is
+// visible; it then calls pdl_trigger() so that the next kernel's CTAs may be
+// scheduled while this one runs (they block in their own pdl_wait()).  A CTA
+// touches no global memory before pdl_wait().
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Launches `kernel` on `s` with programmatic stream serialization allowed.
+template <class... Params, class... Args>
+cudaError_t launch_pdl(void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t s, Args &&...args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 constexpr int kMaxN = 1024;     // experts
 constexpr int kMaxK = 16;       // top-k and warm-up k0
@@ -78,11 +107,11 @@ struct RouteArgs {
 cudaError_t launch_route(const RouteArgs &a, cudaStream_t s);
 cudaError_t launch_router_logits(const uint16_t *x, const float *Wg, float *h, int B, int N,
                                  int d, cudaStream_t s);
-cudaError_t launch_gather(const uint16_t *x, const int32_t *perm, const Meta *meta,
-                          uint16_t *xp, int max_pairs, int d, int k, cudaStream_t s);
 cudaError_t launch_combine(const float *out, const int32_t *pos, const float *w,
                            const Meta *meta, uint16_t *y, int B, int d, int k,
                            cudaStream_t s);
+cudaError_t launch_gather(const uint16_t *x, const int32_t *perm, const Meta *meta,
+                          uint16_t *xp, int max_pairs, int d, int k, cudaStream_t s);
 
 struct FfnArgs {
   const uint16_t *W_gate, *W_up, *W_down;
@@ -100,6 +129,6 @@ struct FfnArgs {
 cudaError_t launch_ffn_gate_up(const FfnArgs &a, cudaStream_t s);
 cudaError_t launch_ffn_down(const FfnArgs &a, cudaStream_t s);
 size_t ffn_part_bytes(int n_sms);
-size_t ffn_cnt_words(int max_tiles, int d, int F);
+size_t ffn_cnt_words(int max_tiles, int B, int d, int F);
 
 }  // namespace xs
