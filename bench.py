@@ -59,6 +59,7 @@ def parse_args(argv=None):
     ap.add_argument("--workload", default="dsr1", choices=sorted(W.WORKLOADS))
     ap.add_argument("--B", type=int, default=None)
     ap.add_argument("--N", type=int, default=None, help="override the expert count (smaller profiling cases)")
+    ap.add_argument("--F", type=int, default=None, help="override d_ff (smaller profiling cases)")
     ap.add_argument("--budget", type=int, default=None)
     ap.add_argument("--k0", type=int, default=None)
     ap.add_argument("--mode", default=None, choices=sorted(W.MODES))
@@ -74,6 +75,8 @@ def workload_from_args(args) -> W.Workload:
         kw["B"] = args.B
     if args.N is not None:
         kw["N"] = args.N
+    if args.F is not None:
+        kw["F"] = args.F
     if args.budget is not None:
         kw["budget"] = args.budget
     if args.k0 is not None:

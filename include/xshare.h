@@ -200,6 +200,15 @@ int xshare_moe_forward_profiled(const uint16_t *x, const float *W_g, const uint1
 /* Name of stage i of xshare_moe_forward (e.g. "router"), or "" if out of range. */
 const char *xshare_stage_name(int i);
 
+/* Self-test of the library's failure reporting (no counterpart in the paper).
+ * Launches one kernel that waits, through the same bounded wait every
+ * pipeline wait of the library uses, on a barrier that nothing arrives at.
+ * After `budget_ns` nanoseconds (1 .. 2e9) the wait gives up; the kernel
+ * writes XS_DEV_TIMEOUT to stats->status, the milliseconds it waited to
+ * stats->reserved[0], and returns, leaving the CUDA context usable.
+ * stats: device pointer (not NULL).  Asynchronous on `stream`. */
+int xshare_selftest_wait_timeout(xs_stats *stats, uint64_t budget_ns, xs_stream_t stream);
+
 /* A static string describing an XS_ERR_* or XS_DEV_* code (never NULL). */
 const char *xshare_strerror(int code);
 

@@ -62,6 +62,8 @@ def _load() -> ctypes.CDLL:
     lib.xshare_route_static.restype = I
     lib.xshare_moe_forward_profiled.argtypes = lib.xshare_moe_forward.argtypes + [P]
     lib.xshare_moe_forward_profiled.restype = I
+    lib.xshare_selftest_wait_timeout.argtypes = [P, ctypes.c_uint64, P]
+    lib.xshare_selftest_wait_timeout.restype = I
     lib.xshare_stage_name.argtypes = [I]
     lib.xshare_stage_name.restype = ctypes.c_char_p
     lib.xshare_strerror.argtypes = [I]
@@ -191,6 +193,13 @@ def xshare_moe_forward(x: torch.Tensor, W_g: torch.Tensor, W_gate: torch.Tensor,
             ev.record()   # torch creates the CUDA event lazily
         handles[i] = ev.cuda_event
     _check(LIB.xshare_moe_forward_profiled(*args, handles), "xshare_moe_forward_profiled")
+
+
+def xshare_selftest_wait_timeout(stats: torch.Tensor, budget_ns: int, stream=None) -> None:
+    """Run the bounded-wait self-test kernel; see xshare.h."""
+    _check(LIB.xshare_selftest_wait_timeout(_ptr(stats, torch.int32, "stats", STATS_WORDS),
+                                            int(budget_ns), _stream(stream)),
+           "xshare_selftest_wait_timeout")
 
 
 def stats_dict(stats: torch.Tensor) -> dict:

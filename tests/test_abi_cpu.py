@@ -28,7 +28,8 @@ def declared_functions():
 
 def test_header_declares_the_boundary():
     assert declared_functions() == ["xshare_moe_forward", "xshare_moe_forward_profiled",
-                                    "xshare_route", "xshare_route_static", "xshare_stage_name",
+                                    "xshare_route", "xshare_route_static",
+                                    "xshare_selftest_wait_timeout", "xshare_stage_name",
                                     "xshare_strerror",
                                     "xshare_workspace_size"]
 
