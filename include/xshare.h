@@ -162,7 +162,7 @@ int xshare_moe_forward(const uint16_t *x, const float *W_g, const uint16_t *W_ga
  * device).  Neither can hand xshare_route a workspace.
  *
  * Same arguments and results as xshare_route, minus the workspace.  The
- * scratch is a fixed array inside the library's device code (about 220 KB
+ * scratch is a fixed array inside the library's device code (about 420 KB
  * on every GPU that loads the library, held until the process exits), so:
  *   - B is limited to 1024 tokens (N <= 1024 and k <= 16 as elsewhere); a
  *     larger B returns XS_ERR_SHAPE and launches nothing;
@@ -170,8 +170,9 @@ int xshare_moe_forward(const uint16_t *x, const float *W_g, const uint16_t *W_ga
  *     cudaGetSymbolAddress; make that first call before any stream capture;
  *   - every call on a device uses the same array, so calls that can overlap
  *     on the GPU (different streams, or different host threads) race and
- *     must be ordered by the caller.  Nothing in the array needs clearing
- *     between calls: the kernel writes each scratch word before reading it.
+ *     must be ordered by the caller.  Each call clears the two arrival
+ *     counters it keeps in the array (a cudaMemsetAsync on `stream`); every
+ *     other scratch word is written before it is read.
  * Allocates nothing (no cudaMalloc, cudaFree or allocating library call). */
 int xshare_route_static(const float *scores, int B, int N, int k, int budget, int mode,
                         const xs_route_params *prm, uint8_t *sel_mask, int32_t *topk_ids,
@@ -179,9 +180,10 @@ int xshare_route_static(const float *scores, int B, int N, int k, int budget, in
                         int32_t *expert_offsets, int32_t *perm, xs_stream_t stream);
 
 /* Kernel stages of xshare_moe_forward, in launch order: router logits,
- * selection (softmax, Algorithms 2-6, refinement, permutation), token
- * gather, SwiGLU gate/up, SwiGLU down, weighted combine. */
-#define XS_N_STAGES 6
+ * selection (softmax, ranking, column scores, Algorithms 2-6), refinement
+ * and permutation, token gather, SwiGLU gate/up, SwiGLU down, weighted
+ * combine. */
+#define XS_N_STAGES 7
 
 /* xshare_moe_forward that also records CUDA events on `stream` between its
  * kernel launches, so a caller can time each stage on the launching stream:

@@ -92,6 +92,9 @@ RouteArgs route_args(const Plan &pl, void *ws, int B, int N, int k, int budget, 
   a.pos = at<int32_t>(ws, pl.pos);
   a.tiles = at<Tile>(ws, pl.tiles);
   a.meta = at<Meta>(ws, pl.meta);
+  a.chunk_col = at<float>(ws, pl.chunk_col);
+  a.chunk_marks = at<uint8_t>(ws, pl.chunk_marks);
+  a.done = at<int32_t>(ws, pl.done);
   return a;
 }
 
@@ -121,6 +124,10 @@ Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms) {
   pl.pos = take((size_t)B * k * 4);
   pl.tiles = take((size_t)pl.max_tiles * sizeof(Tile));
   pl.meta = take(sizeof(Meta));
+  const int chunks = (B + kChunk - 1) / kChunk;
+  pl.chunk_col = take((size_t)chunks * N * 4);
+  pl.chunk_marks = take((size_t)chunks * 2 * N);
+  pl.done = take(4 * sizeof(int32_t));
   if (with_ffn) {
     pl.xp = take((size_t)pl.max_pairs * d * 2);
     pl.act = take((size_t)pl.max_pairs * F * 2);
@@ -170,12 +177,13 @@ extern "C" int xshare_route(const float *scores, int B, int N, int k, int budget
   a.offsets_out = expert_offsets;
   a.perm_out = perm;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(a.done, 0, 2 * sizeof(int32_t), s) != cudaSuccess) return XS_ERR_CUDA;
   return launch_route(a, s) == cudaSuccess ? XS_OK : XS_ERR_CUDA;
 }
 
 namespace {
 
-const char *const kStageNames[XS_N_STAGES] = {"router", "select", "gather", "ffn_gate_up",
+const char *const kStageNames[XS_N_STAGES] = {"router", "select", "refine", "gather", "ffn_gate_up",
                                               "ffn_down", "combine"};
 
 int forward_impl(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
@@ -235,15 +243,17 @@ int forward_impl(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
            cudaEventRecord(reinterpret_cast<cudaEvent_t>(events[i]), s) == cudaSuccess;
   };
   if (!mark(0)) return XS_ERR_CUDA;
-  if (launch_router_logits(x, W_g, h, B, N, d, s) != cudaSuccess || !mark(1)) return XS_ERR_CUDA;
-  if (launch_route(a, s) != cudaSuccess || !mark(2)) return XS_ERR_CUDA;
+  if (launch_router_logits(x, W_g, h, B, N, d, a.done, s) != cudaSuccess || !mark(1))
+    return XS_ERR_CUDA;
+  a.events = events ? events + 2 : nullptr;  // between the selection and refinement kernels
+  if (launch_route(a, s) != cudaSuccess || !mark(3)) return XS_ERR_CUDA;
   if (launch_gather(x, a.perm, a.meta, const_cast<uint16_t *>(f.xp), pl.max_pairs, d, k, s) !=
           cudaSuccess ||
-      !mark(3))
+      !mark(4))
     return XS_ERR_CUDA;
-  if (launch_ffn_gate_up(f, s) != cudaSuccess || !mark(4)) return XS_ERR_CUDA;
-  if (launch_ffn_down(f, s) != cudaSuccess || !mark(5)) return XS_ERR_CUDA;
-  if (launch_combine(f.out, a.pos, a.w, a.meta, y, B, d, k, s) != cudaSuccess || !mark(6))
+  if (launch_ffn_gate_up(f, s) != cudaSuccess || !mark(5)) return XS_ERR_CUDA;
+  if (launch_ffn_down(f, s) != cudaSuccess || !mark(6)) return XS_ERR_CUDA;
+  if (launch_combine(f.out, a.pos, a.w, a.meta, y, B, d, k, s) != cudaSuccess || !mark(7))
     return XS_ERR_CUDA;
   return XS_OK;
 }

@@ -170,57 +170,254 @@ __device__ __forceinline__ void block_scan3(int (&v)[3], int (&tot)[3], int *s_t
   __syncthreads();
 }
 
-// The whole selection in one CTA (steps a2-a7):
-//   1. per token (one warp each): dense softmax of the logits (or the given
-//      scores), then its ranked top-max(k, k0) over E, which marks the plain
-//      top-k union and the warm-up set S_0;
-//   2. canonical column sums (one thread per expert) and, for HIER, the
-//      per-request selections of Algorithm 3 (one warp per request);
-//   3. the budgeted selection: BATCH and the batch step of HIER rank the
-//      column scores outside the base set in one warp; GROUP ranks each
-//      group's scores in its own warp (Algorithm 5's rounds in closed form);
-//   4. per token the top-k' inside S with renormalised weights, counting the
-//      pairs per expert on the way;
-//   5. prefix sums, FFN tiles, and the stable scatter of the pairs.
-// The score matrix and the ids are staged in shared memory when they fit.
+// Selection is split over two kernels whose CTAs each own one chunk of 32
+// tokens (the canonical summation chunk, so column sums stay bit-identical to
+// a single-pass evaluation):
+//
+//   score_kernel  (a2, a3, a4, part of a5): per token (one warp each) the
+//       dense softmax of the logits (or the given scores) and its ranked
+//       top-max(k, k0) over E; the chunk's column-sum tree; the chunk's
+//       warm-up and plain top-k union marks; for HIER, Algorithm 3 for every
+//       request inside the chunk.  The CTA that finishes last adds the chunk
+//       sums left to right, merges the marks and runs the budgeted selection
+//       (a5): BATCH and the batch step of HIER rank the column scores outside
+//       the base set in one warp; GROUP ranks each group in its own warp
+//       (Algorithm 5's rounds in closed form).
+//   refine_kernel (a6, a7): per token the top-k' inside S with renormalised
+//       weights.  The CTA that finishes last counts the pairs per expert,
+//       takes the prefix sums, writes the FFN tiles and scatters the pairs
+//       stably by expert.
+//
+// "Last to finish" uses an arrival counter per kernel, cleared before the
+// first kernel of the call: every CTA writes its results, fences, and bumps
+// the counter; the CTA that sees the final count continues alone.  No CTA
+// waits for another.
+
+__device__ __forceinline__ int chunk_count(int B) { return (B + kChunk - 1) / kChunk; }
+
+// Selected set statistics: |S|, plain top-k union, max group load.
+__device__ __forceinline__ void selection_stats(const RouteArgs &a, const uint8_t *s_mask,
+                                                const uint8_t *s_union, int *s_gl, int &nsel,
+                                                int &n_union, int &maxload) {
+  const int tid = threadIdx.x, N = a.N;
+  const int G = a.G >= 1 ? a.G : 1, size = N / G;
+  for (int g = tid; g < G; g += blockDim.x) s_gl[g] = 0;
+  __syncthreads();
+  for (int j = tid; j < N; j += blockDim.x)
+    if (s_mask[j]) atomicAdd(&s_gl[j / size], 1);
+  nsel = __syncthreads_count(tid < N && s_mask[tid]);
+  n_union = __syncthreads_count(tid < N && s_union[tid]);
+  int best = 0;
+  for (int g = tid; g < G; g += blockDim.x) best = max(best, s_gl[g]);
+  best = __reduce_max_sync(kFull, best);
+  if ((tid & 31) == 0) atomicMax(&s_gl[kMaxN], best);
+  __syncthreads();
+  maxload = s_gl[kMaxN];
+}
+
+// Per token t in [t_begin, t_end), one warp each: Top k'(G_t, S) with the
+// renormalised weights (a6); row(t) points at the token's scores.
+template <int kQ, class Row>
+__device__ __forceinline__ void refine_tokens(const RouteArgs &a, const uint8_t *s_mask,
+                                              int t_begin, int t_end, int kp, Row row,
+                                              int32_t *ids_s = nullptr) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  const int N = a.N, k = a.k;
+  for (int t = t_begin + warp; t < t_end; t += nwarps) {
+    const float *prow = row(t);
+    LaneList<kQ> L;
+    lane_load<kQ>(L, 0, N, lane, [&](int, int j) { return prow[j]; },
+                  [&](int, int j) { return s_mask[j] != 0; });
+    lane_sort<kQ>(L);
+    int my_id = -1;  // lane s keeps slot s
+    float my_v = 0.f;
+    float D = 0.f;
+    const int got = lane_take<kQ>(L, kp, [&](int r, int id, float v) {
+      if (lane == r) {
+        my_id = id;
+        my_v = v;
+      }
+      D = __fadd_rn(D, v);  // slot order, identical on every lane
+    });
+    if (lane < k) {
+      float wv = 0.f;
+      if (lane < got) wv = (D > 0.f) ? __fdiv_rn(my_v, D) : __fdiv_rn(1.f, (float)got);
+      a.ids[(size_t)t * k + lane] = (lane < got) ? my_id : -1;
+      if (ids_s) ids_s[(t - t_begin) * k + lane] = (lane < got) ? my_id : -1;
+      a.w[(size_t)t * k + lane] = wv;
+    }
+  }
+}
+
+struct PermSmem {
+  int32_t *counts, *cursor, *chunk, *tmp, *scal, *wcnt;  // wcnt: [32][N] (N <= kScatterMaxN)
+  const int32_t *ids;  // nullable: the ids in shared memory (else read from global)
+};
+
+// Counting sort of all pairs by expert, stable in (token, slot) (a7), the FFN
+// tiles and the statistics.  One CTA, once every token's ids are written and
+// visible; the meta block already holds the selection's fields.
+__device__ void build_permutation(const RouteArgs &a, PermSmem sm) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int nwarps = blockDim.x >> 5;
+  const int B = a.B, N = a.N, k = a.k;
+  const int P = B * k;
+  for (int j = tid; j < N; j += blockDim.x) sm.counts[j] = 0;
+  __syncthreads();
+  for (int q = tid; q < P; q += blockDim.x) {
+    const int e = sm.ids ? sm.ids[q] : __ldcg(a.ids + q);
+    if ((unsigned)e < (unsigned)N) atomicAdd(&sm.counts[e], 1);
+  }
+  __syncthreads();
+  {
+    const int cnt = tid < N ? sm.counts[tid] : 0;
+    int v[3] = {cnt, (cnt + kTileTok - 1) / kTileTok, cnt > 0 ? 1 : 0}, tot[3];
+    block_scan3(v, tot, sm.tmp);
+    if (tid < N) {
+      sm.cursor[tid] = v[0];
+      a.counts[tid] = cnt;
+      a.offsets[tid] = v[0];
+      if (a.counts_out) a.counts_out[tid] = cnt;
+      if (a.offsets_out) a.offsets_out[tid] = v[0];
+      for (int tt = 0; tt * kTileTok < cnt; ++tt) {
+        Tile tl;
+        tl.expert = tid;
+        tl.row0 = v[0] + tt * kTileTok;
+        tl.ntok = min(kTileTok, cnt - tt * kTileTok);
+        tl.pad = 0;
+        a.tiles[v[1] + tt] = tl;
+      }
+    }
+    if (tid == 0) {
+      a.offsets[N] = tot[0];
+      if (a.offsets_out) a.offsets_out[N] = tot[0];
+      sm.scal[1] = tot[0];  // pairs
+      sm.scal[2] = tot[1];  // tiles
+      sm.scal[3] = tot[2];  // used experts
+    }
+  }
+  __syncthreads();
+  const unsigned lt = (1u << lane) - 1u;
+  if (N <= kScatterMaxN) {
+    // Chunks of blockDim pairs: rank inside a warp by match_any, then an
+    // exclusive prefix over the warps of the chunk for every expert.
+    for (int base = 0; base < P; base += blockDim.x) {
+      for (int i = tid; i < 32 * N; i += blockDim.x) sm.wcnt[i] = 0;
+      const int q = base + tid;
+      int e = (q < P) ? (sm.ids ? sm.ids[q] : __ldcg(a.ids + q)) : -1;
+      if ((unsigned)e >= (unsigned)N) e = -1;
+      const unsigned peers = __match_any_sync(kFull, e);
+      const int rank = __popc(peers & lt);
+      __syncthreads();
+      if (e >= 0 && rank == 0) sm.wcnt[warp * N + e] = __popc(peers);
+      __syncthreads();
+      if (tid < N) {
+        int run = 0;
+        for (int w = 0; w < nwarps; ++w) {
+          const int x = sm.wcnt[w * N + tid];
+          sm.wcnt[w * N + tid] = run;
+          run += x;
+        }
+        sm.chunk[tid] = run;
+      }
+      __syncthreads();
+      if (e >= 0) {
+        const int r = sm.cursor[e] + sm.wcnt[warp * N + e] + rank;
+        a.perm[r] = q;
+        a.pos[q] = r;
+        if (a.perm_out) a.perm_out[r] = q;
+      } else if (q < P) {
+        a.pos[q] = -1;
+      }
+      __syncthreads();
+      if (tid < N) sm.cursor[tid] += sm.chunk[tid];
+      __syncthreads();
+    }
+  } else if (warp == 0) {
+    for (int base = 0; base < P; base += 32) {
+      const int q = base + lane;
+      int e = (q < P) ? (sm.ids ? sm.ids[q] : __ldcg(a.ids + q)) : -1;
+      if ((unsigned)e >= (unsigned)N) e = -1;
+      const unsigned peers = __match_any_sync(kFull, e);
+      const int rank = __popc(peers & lt);
+      const int old = (e >= 0) ? sm.cursor[e] : 0;
+      __syncwarp();
+      if (e >= 0) {
+        const int r = old + rank;
+        a.perm[r] = q;
+        a.pos[q] = r;
+        if (a.perm_out) a.perm_out[r] = q;
+        if (rank == 0) sm.cursor[e] = old + __popc(peers);
+      } else if (q < P) {
+        a.pos[q] = -1;
+      }
+      __syncwarp();
+    }
+  }
+  if (tid == 0) {
+    Meta m = *a.meta;
+    m.n_pairs = sm.scal[1];  // == B * kp unless scores were non-finite
+    m.n_tiles = sm.scal[2];
+    m.n_used = sm.scal[3];
+    *a.meta = m;
+    if (a.stats) {
+      xs_stats st;
+      st.n_selected = m.n_selected;
+      st.n_used = m.n_used;
+      st.union_topk = m.union_topk;
+      st.max_group_load = m.max_group_load;
+      st.n_pairs = m.n_pairs;
+      st.status = 0;
+      st.reserved[0] = st.reserved[1] = 0;
+      *a.stats = st;
+    }
+  }
+}
+
 template <int kQ>
-__global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
-  extern __shared__ float dsm[];
-  __shared__ uint8_t s_mask[kMaxN];   // S
-  __shared__ uint8_t s_base[kMaxN];   // S_0 (or the union of the S_r for HIER)
-  __shared__ uint8_t s_union[kMaxN];  // union of plain top-k
-  __shared__ float s_col[kMaxN];      // batch column scores
-  __shared__ int32_t s_counts[kMaxN];
+__global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
+  extern __shared__ float ps[];         // [32][N] scores of the chunk's tokens (+ [32][N] ints)
+  __shared__ uint8_t s_mask[kMaxN];     // S (selection step)
+  __shared__ uint8_t s_base[kMaxN];     // chunk marks: S_0 (or S_r for HIER); merged later
+  __shared__ uint8_t s_union[kMaxN];    // chunk marks: plain top-k union; merged later
+  __shared__ float s_col[kMaxN];
+  __shared__ int32_t s_gl[kMaxN + 1];
+  __shared__ int32_t s_top[kChunk][kMaxK];
+  __shared__ int32_t s_scal[4];
+  __shared__ int32_t s_counts[kMaxN];   // permutation, when it runs in this kernel
   __shared__ int32_t s_cursor[kMaxN];
-  __shared__ int32_t s_avail[kMaxN];
+  __shared__ int32_t s_chunk[kMaxN];
   __shared__ int32_t s_tmp[200];
-  __shared__ int32_t s_scal[8];       // 0:R* 1:max group load 2:|U| 3:tiles 4:pairs
 
   pdl_wait();
   pdl_trigger();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nwarps = blockDim.x >> 5;
   const int B = a.B, N = a.N, k = a.k;
-  const int kk = max(k, a.k0);  // ranked list length per token
+  const int C = chunk_count(B), c = blockIdx.x;
+  const int t0 = c * kChunk, nt = min(kChunk, B - t0);
+  const int kk = max(k, a.k0);
   const bool hier = a.mode == XS_MODE_HIER;
-  float *ps = a.p_smem ? dsm : nullptr;
-  int32_t *ids_s = a.ids_smem ? reinterpret_cast<int32_t *>(dsm + (a.p_smem ? B * N : 0)) : nullptr;
-  // Per-warp expert counts of the parallel scatter: [32][N] after p and ids.
-  int32_t *s_wcnt = reinterpret_cast<int32_t *>(dsm) + (a.p_smem ? B * N : 0) + (a.ids_smem ? B * k : 0);
-  const float *P = ps ? ps : a.p;
+  // HIER requests that lie inside one chunk are selected here (Algorithm 3);
+  // otherwise the selection step does it from the full score matrix.
+  const bool hier_here = hier && a.T <= kChunk && kChunk % a.T == 0;
 
   for (int j = tid; j < N; j += blockDim.x) {
-    s_mask[j] = 0;
     s_base[j] = 0;
     s_union[j] = 0;
-    s_counts[j] = 0;
   }
   if (a.zero_words != nullptr)
-    for (int i = tid; i < a.zero_count; i += blockDim.x) a.zero_words[i] = 0;
+    for (int i = c * blockDim.x + tid; i < a.zero_count; i += C * blockDim.x) a.zero_words[i] = 0;
   __syncthreads();
 
-  // ---- 1. scores (a2) and per-token ranking over E (a3) ----
-  for (int t = warp; t < B; t += nwarps) {
+  // ---- per token: scores (a2) and ranking over E (a3) ----
+  for (int w = warp; w < kChunk; w += nwarps) {
+    float *prow_s = ps + w * N;
+    if (w >= nt) {  // zero rows pad the last chunk's tree
+      for (int j = lane; j < N; j += 32) prow_s[j] = 0.f;
+      continue;
+    }
+    const int t = t0 + w;
     float vals[kQ];
     if (a.logits != nullptr) {
       const float *hrow = a.logits + (size_t)t * N;
@@ -247,7 +444,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
         if (j < N) {
           vals[q] = __fdiv_rn(vals[q], sum);
           a.p[(size_t)t * N + j] = vals[q];
-          if (ps) ps[t * N + j] = vals[q];
+          prow_s[j] = vals[q];
         }
       }
     } else {
@@ -255,7 +452,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
       for (int q = 0; q < kQ; ++q) {
         const int j = lane + 32 * q;
         vals[q] = (j < N) ? a.p[(size_t)t * N + j] : 0.f;
-        if (ps && j < N) ps[t * N + j] = vals[q];
+        if (j < N) prow_s[j] = vals[q];
       }
     }
     LaneList<kQ> L;
@@ -267,6 +464,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
       if (lane == 0) {
         if (r < k) s_union[id] = 1;
         if (r < a.k0) {
+          s_top[w][r] = id;
           if (hier)
             top[r] = id;
           else
@@ -277,31 +475,42 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
   }
   __syncthreads();
 
-  // ---- 2. batch column scores (a4) ----
-  for (int j = tid; j < N; j += blockDim.x) s_col[j] = canonical_sum(P, N, j, 0, B);
+  // ---- the chunk's column-sum tree (a4) ----
+  for (int j = tid; j < N; j += blockDim.x) {
+    float v[kChunk];
+#pragma unroll
+    for (int l = 0; l < kChunk; ++l) v[l] = ps[l * N + j];
+#pragma unroll
+    for (int o = kChunk / 2; o; o >>= 1) {
+#pragma unroll
+      for (int l = 0; l < o; ++l) v[l] = __fadd_rn(v[l], v[l + o]);
+    }
+    if (C == 1)
+      s_col[j] = __fadd_rn(0.f, v[0]);  // one chunk: the batch sum is 0 + the chunk's tree
+    else
+      a.chunk_col[(size_t)c * N + j] = v[0];
+  }
 
-  // ---- 2'. HIER: per-request selection (Algorithm 3), one warp per request ----
-  if (hier) {
-    const int T = a.T, R = B / T;
-    for (int r = warp; r < R; r += nwarps) {
-      const int r0 = r * T, r1 = r0 + T;
+  // ---- HIER: Algorithm 3 for the requests inside this chunk ----
+  if (hier_here) {
+    const int T = a.T;
+    for (int r = warp; r * T < nt; r += nwarps) {
+      const int r0 = r * T, r1 = min(r0 + T, nt);
       float sc[kQ];
       uint32_t excl = 0;
 #pragma unroll
       for (int q = 0; q < kQ; ++q) {
         const int j = lane + 32 * q;
-        sc[q] = (j < N) ? canonical_sum(P, N, j, r0, r1) : 0.f;
+        sc[q] = (j < N) ? canonical_sum(ps, N, j, r0, r1) : 0.f;
       }
-      // S0_r: union of Top k0 over the request's tokens.
       for (int x = r0; x < r1; ++x)
         for (int i = 0; i < a.k0; ++i) {
-          const int e = a.toptok[(size_t)x * kMaxK + i];
+          const int e = s_top[x][i];
           if ((unsigned)e < (unsigned)N && (e & 31) == lane) {
             excl |= 1u << (e >> 5);
             s_base[e] = 1;
           }
         }
-      // S_r = S0_r + Top m_r(scores_r, E \ S0_r).
       LaneList<kQ> L;
       lane_load<kQ>(L, 0, N, lane, [&](int q, int) { return sc[q]; },
                     [&](int q, int) { return ((excl >> q) & 1u) == 0; });
@@ -312,8 +521,69 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
     }
   }
   __syncthreads();
+  if (C > 1) {
+    uint8_t *marks = a.chunk_marks + (size_t)c * 2 * N;
+    for (int j = tid; j < N; j += blockDim.x) {
+      marks[j] = s_base[j];
+      marks[N + j] = s_union[j];
+    }
 
-  // ---- 3. budgeted selection (a5) ----
+    // ---- the last CTA to finish runs the selection ----
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) s_scal[0] = (atomicAdd(&a.done[0], 1) == C - 1) ? 1 : 0;
+    __syncthreads();
+    if (!s_scal[0]) return;
+    __threadfence();
+
+    for (int j = tid; j < N; j += blockDim.x) {
+      float acc = 0.f;
+      uint8_t b = 0, u = 0;
+      for (int cc = 0; cc < C; ++cc) {
+        acc = __fadd_rn(acc, __ldcg(a.chunk_col + (size_t)cc * N + j));
+        const uint8_t *m = a.chunk_marks + (size_t)cc * 2 * N;
+        b |= __ldcg(m + j);
+        u |= __ldcg(m + N + j);
+      }
+      s_col[j] = acc;
+      s_base[j] = b;
+      s_union[j] = u;
+    }
+  }
+  __syncthreads();
+
+  if (hier && !hier_here) {
+    // Requests cross chunk boundaries: Algorithm 3 from the full score matrix.
+    const int T = a.T, R = B / T;
+    for (int r = warp; r < R; r += nwarps) {
+      const int r0 = r * T, r1 = r0 + T;
+      float sc[kQ];
+      uint32_t excl = 0;
+#pragma unroll
+      for (int q = 0; q < kQ; ++q) {
+        const int j = lane + 32 * q;
+        sc[q] = (j < N) ? canonical_sum(a.p, N, j, r0, r1) : 0.f;
+      }
+      for (int x = r0; x < r1; ++x)
+        for (int i = 0; i < a.k0; ++i) {
+          const int e = __ldcg(a.toptok + (size_t)x * kMaxK + i);
+          if ((unsigned)e < (unsigned)N && (e & 31) == lane) {
+            excl |= 1u << (e >> 5);
+            s_base[e] = 1;
+          }
+        }
+      LaneList<kQ> L;
+      lane_load<kQ>(L, 0, N, lane, [&](int q, int) { return sc[q]; },
+                    [&](int q, int) { return ((excl >> q) & 1u) == 0; });
+      lane_sort<kQ>(L);
+      lane_take<kQ>(L, a.m_r, [&](int, int id, float) {
+        if (lane == 0) s_base[id] = 1;
+      });
+    }
+    __syncthreads();
+  }
+
+  // ---- budgeted selection (a5) ----
   for (int j = tid; j < N; j += blockDim.x) s_mask[j] = s_base[j];
   __syncthreads();
   if (a.mode == XS_MODE_TOPK) {
@@ -325,27 +595,27 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
     const int G = a.G, size = N / G;
     const int n_base = __syncthreads_count(tid < N && s_base[tid]);
     for (int g = warp; g < G; g += nwarps) {
-      int c = 0;
-      for (int j = g * size + lane; j < (g + 1) * size; j += 32) c += s_base[j] ? 0 : 1;
-      c = __reduce_add_sync(kFull, c);
-      if (lane == 0) s_avail[g] = c;
+      int cnt = 0;
+      for (int j = g * size + lane; j < (g + 1) * size; j += 32) cnt += s_base[j] ? 0 : 1;
+      cnt = __reduce_add_sync(kFull, cnt);
+      if (lane == 0) s_gl[g] = cnt;
     }
     __syncthreads();
     if (tid == 0) {
       int maxav = 0;
-      for (int g = 0; g < G; ++g) maxav = max(maxav, s_avail[g]);
+      for (int g = 0; g < G; ++g) maxav = max(maxav, s_gl[g]);
       const long long target = (long long)a.m_g * G;
       int R = 0;
       for (;;) {
         long long tot = n_base;
-        for (int g = 0; g < G; ++g) tot += min(R, s_avail[g]);
+        for (int g = 0; g < G; ++g) tot += min(R, s_gl[g]);
         if (tot >= target || R >= maxav) break;
         ++R;
       }
-      s_scal[0] = R;
+      s_scal[1] = R;
     }
     __syncthreads();
-    const int R = s_scal[0];
+    const int R = s_scal[1];
     if (R > 0)
       for (int g = warp; g < G; g += nwarps) {
         LaneList<kQ> L;
@@ -363,173 +633,75 @@ __global__ void __launch_bounds__(kRouteThreads, 1) route_kernel(RouteArgs a) {
     lane_load<kQ>(L, 0, N, lane, [&](int, int j) { return s_col[j]; },
                   [&](int, int j) { return s_base[j] == 0; });
     lane_sort<kQ>(L);
-    __syncwarp();
     lane_take<kQ>(L, a.budget, [&](int, int id, float) {
       if (lane == 0) s_mask[id] = 1;
     });
   }
   __syncthreads();
 
-  // ---- statistics ----
-  const int nsel = __syncthreads_count(tid < N && s_mask[tid]);
-  const int n_union = __syncthreads_count(tid < N && s_union[tid]);
-  if (warp == 0) {
-    const int G = a.G >= 1 ? a.G : 1;
-    const int size = N / G;
-    int best = 0;
-    for (int g = lane; g < G; g += 32) {
-      int c = 0;
-      for (int j = g * size; j < (g + 1) * size; ++j) c += s_mask[j];
-      best = max(best, c);
-    }
-    best = __reduce_max_sync(kFull, best);
-    if (lane == 0) s_scal[1] = best;
-  }
+  int nsel, n_union, maxload;
+  if (tid == 0) s_gl[kMaxN] = 0;
+  selection_stats(a, s_mask, s_union, s_gl, nsel, n_union, maxload);
   for (int j = tid; j < N; j += blockDim.x) a.mask[j] = s_mask[j];
-  const int kp = min(k, nsel);
-
-  // ---- 4. refinement (a6): Top k'(G_i, S), renormalised weights, pair counts ----
-  for (int t = warp; t < B; t += nwarps) {
-    LaneList<kQ> L;
-    const float *prow = P + (size_t)t * N;
-    lane_load<kQ>(L, 0, N, lane, [&](int, int j) { return prow[j]; },
-                  [&](int, int j) { return s_mask[j] != 0; });
-    lane_sort<kQ>(L);
-    int my_id = -1;  // lane s keeps slot s
-    float my_v = 0.f;
-    float D = 0.f;
-    const int got = lane_take<kQ>(L, kp, [&](int r, int id, float v) {
-      if (lane == r) {
-        my_id = id;
-        my_v = v;
-      }
-      D = __fadd_rn(D, v);  // slot order, identical on every lane
-    });
-    if (lane < k) {
-      float wv = 0.f;
-      if (lane < got) wv = (D > 0.f) ? __fdiv_rn(my_v, D) : __fdiv_rn(1.f, (float)got);
-      const int id = (lane < got) ? my_id : -1;
-      a.ids[(size_t)t * k + lane] = id;
-      a.w[(size_t)t * k + lane] = wv;
-      if (ids_s) ids_s[t * k + lane] = id;
-      if (id >= 0) atomicAdd(&s_counts[id], 1);
-    }
-  }
-  __syncthreads();
-
-  // ---- 5. permutation (a7): counting sort by expert, stable in (token, slot) ----
-  {
-    const int c = tid < N ? s_counts[tid] : 0;
-    int v[3] = {c, (c + kTileTok - 1) / kTileTok, c > 0 ? 1 : 0}, tot[3];
-    block_scan3(v, tot, s_tmp);
-    if (tid < N) {
-      s_cursor[tid] = v[0];
-      a.counts[tid] = c;
-      a.offsets[tid] = v[0];
-      if (a.counts_out) a.counts_out[tid] = c;
-      if (a.offsets_out) a.offsets_out[tid] = v[0];
-      for (int tt = 0; tt * kTileTok < c; ++tt) {
-        Tile tl;
-        tl.expert = tid;
-        tl.row0 = v[0] + tt * kTileTok;
-        tl.ntok = min(kTileTok, c - tt * kTileTok);
-        tl.pad = 0;
-        a.tiles[v[1] + tt] = tl;
-      }
-    }
-    if (tid == 0) {
-      a.offsets[N] = tot[0];
-      if (a.offsets_out) a.offsets_out[N] = tot[0];
-      s_scal[2] = tot[2];
-      s_scal[3] = tot[1];
-      s_scal[4] = tot[0];
-    }
-  }
-  __syncthreads();
-  const int P2 = B * k;
-  const int32_t *ids = ids_s ? ids_s : a.ids;
-  if (N <= kScatterMaxN) {
-    // Chunks of blockDim pairs: rank inside a warp by match_any, then an
-    // exclusive prefix over the warps of the chunk for every expert.
-    const unsigned lt = (1u << lane) - 1u;
-    for (int base = 0; base < P2; base += blockDim.x) {
-      for (int i = tid; i < 32 * N; i += blockDim.x) s_wcnt[i] = 0;
-      const int q = base + tid;
-      int e = (q < P2) ? ids[q] : -1;
-      if ((unsigned)e >= (unsigned)N) e = -1;
-      const unsigned peers = __match_any_sync(kFull, e);
-      const int rank = __popc(peers & lt);
-      __syncthreads();
-      if (e >= 0 && rank == 0) s_wcnt[warp * N + e] = __popc(peers);
-      __syncthreads();
-      if (tid < N) {
-        int run = 0;
-        for (int w = 0; w < nwarps; ++w) {
-          const int x = s_wcnt[w * N + tid];
-          s_wcnt[w * N + tid] = run;
-          run += x;
-        }
-        s_avail[tid] = run;
-      }
-      __syncthreads();
-      if (e >= 0) {
-        const int r = s_cursor[e] + s_wcnt[warp * N + e] + rank;
-        a.perm[r] = q;
-        a.pos[q] = r;
-        if (a.perm_out) a.perm_out[r] = q;
-      } else if (q < P2) {
-        a.pos[q] = -1;
-      }
-      __syncthreads();
-      if (tid < N) s_cursor[tid] += s_avail[tid];
-      __syncthreads();
-    }
-  } else if (warp == 0) {
-    const unsigned lt = (1u << lane) - 1u;
-    for (int base = 0; base < P2; base += 32) {
-      const int q = base + lane;
-      int e = (q < P2) ? ids[q] : -1;
-      if ((unsigned)e >= (unsigned)N) e = -1;
-      const unsigned peers = __match_any_sync(kFull, e);
-      const int rank = __popc(peers & lt);
-      const int old = (e >= 0) ? s_cursor[e] : 0;
-      __syncwarp();
-      if (e >= 0) {
-        const int r = old + rank;
-        a.perm[r] = q;
-        a.pos[q] = r;
-        if (a.perm_out) a.perm_out[r] = q;
-        if (rank == 0) s_cursor[e] = old + __popc(peers);
-      } else if (q < P2) {
-        a.pos[q] = -1;
-      }
-      __syncwarp();
-    }
-  }
   if (tid == 0) {
     Meta m;
-    m.n_pairs = s_scal[4];  // == B * kp unless scores were non-finite
-    m.n_tiles = s_scal[3];
-    m.kprime = kp;
-    m.n_selected = nsel;
-    m.n_used = s_scal[2];
-    m.union_topk = n_union;
-    m.max_group_load = s_scal[1];
-    m.status = 0;
     for (int i = 0; i < 8; ++i) m.pad[i] = 0;
+    m.n_pairs = 0;
+    m.n_tiles = 0;
+    m.kprime = min(k, nsel);
+    m.n_selected = nsel;
+    m.n_used = 0;
+    m.union_topk = n_union;
+    m.max_group_load = maxload;
+    m.status = 0;
     *a.meta = m;
-    if (a.stats) {
-      xs_stats st;
-      st.n_selected = nsel;
-      st.n_used = s_scal[2];
-      st.union_topk = n_union;
-      st.max_group_load = s_scal[1];
-      st.n_pairs = s_scal[4];
-      st.status = 0;
-      st.reserved[0] = st.reserved[1] = 0;
-      *a.stats = st;
-    }
   }
+  if (!a.fuse_refine) return;
+  // Small batches: refinement and permutation in this CTA too (no second
+  // kernel); this chunk's scores are still in shared memory.
+  __syncthreads();
+  int32_t *ids_s = C == 1 ? &s_top[0][0] : nullptr;  // one chunk: ids stay in shared memory
+  refine_tokens<kQ>(
+      a, s_mask, 0, B, min(k, nsel),
+      [&](int t) -> const float * {
+        return (t >= t0 && t < t0 + nt) ? ps + (t - t0) * N : a.p + (size_t)t * N;
+      },
+      ids_s);
+  if (C > 1) __threadfence();
+  __syncthreads();
+  build_permutation(a, PermSmem{s_counts, s_cursor, s_chunk, s_tmp, s_scal,
+                                reinterpret_cast<int32_t *>(ps + kChunk * N), ids_s});
+}
+
+template <int kQ>
+__global__ void __launch_bounds__(kRouteThreads, 1) refine_kernel(RouteArgs a) {
+  extern __shared__ int32_t s_wcnt[];   // [32][N] per-warp counts of the scatter (N <= 256)
+  __shared__ uint8_t s_mask[kMaxN];
+  __shared__ int32_t s_counts[kMaxN];
+  __shared__ int32_t s_cursor[kMaxN];
+  __shared__ int32_t s_chunk[kMaxN];
+  __shared__ int32_t s_tmp[200];
+  __shared__ int32_t s_scal[4];
+
+  pdl_wait();
+  pdl_trigger();
+  const int tid = threadIdx.x;
+  const int B = a.B, N = a.N;
+  const int C = chunk_count(B), c = blockIdx.x;
+  const int t0 = c * kChunk, nt = min(kChunk, B - t0);
+  const int kp = a.meta->kprime;
+  for (int j = tid; j < N; j += blockDim.x) s_mask[j] = a.mask[j];
+  __syncthreads();
+  refine_tokens<kQ>(a, s_mask, t0, t0 + nt, kp, [&](int t) { return a.p + (size_t)t * N; });
+
+  // ---- the last CTA to finish builds the permutation (a7) ----
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) s_scal[0] = (atomicAdd(&a.done[1], 1) == C - 1) ? 1 : 0;
+  __syncthreads();
+  if (!s_scal[0]) return;
+  __threadfence();
+  build_permutation(a, PermSmem{s_counts, s_cursor, s_chunk, s_tmp, s_scal, s_wcnt, nullptr});
 }
 
 // ---- a1: router logits h = W_g x, fp32.
@@ -560,10 +732,11 @@ __device__ __forceinline__ void rt_load(const uint2 *__restrict__ xbase,
 
 __global__ void __launch_bounds__(kRtWarps * 32) router_logits_kernel(
     const uint16_t *__restrict__ x, const float *__restrict__ Wg, float *__restrict__ h, int B,
-    int N, int d) {
+    int N, int d, int32_t *__restrict__ done) {
   __shared__ float red[kRtWarps][kRtOut];
   pdl_wait();
   pdl_trigger();
+  if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x < 2) done[threadIdx.x] = 0;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int e0 = blockIdx.x * kRtExp, t0 = blockIdx.y * kRtTok;
   const int d4 = d / 4;
@@ -676,24 +849,29 @@ __global__ void __launch_bounds__(256) combine_kernel(const float *__restrict__ 
 
 }  // namespace
 
-size_t route_dynamic_smem(int B, int N, int k, bool *p_smem, bool *ids_smem) {
-  const size_t p_bytes = (size_t)B * N * 4, ids_bytes = (size_t)B * k * 4;
-  *p_smem = p_bytes <= kRouteSmemP;
-  *ids_smem = ids_bytes <= kRouteSmemIds;
-  const size_t wcnt_bytes = N <= kScatterMaxN ? (size_t)32 * N * 4 : 0;
-  return (*p_smem ? p_bytes : 0) + (*ids_smem ? ids_bytes : 0) + wcnt_bytes;
-}
-
-template <int kMaxQ>
-cudaError_t launch_route_q(RouteArgs a, cudaStream_t s) {
-  bool ps = false, is = false;
-  const size_t dyn = route_dynamic_smem(a.B, a.N, a.k, &ps, &is);
-  a.p_smem = ps ? 1 : 0;
-  a.ids_smem = is ? 1 : 0;
-  cudaError_t e = cudaFuncSetAttribute(route_kernel<kMaxQ>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+template <int kQ>
+cudaError_t launch_route_q(const RouteArgs &a, cudaStream_t s) {
+  const int C = (a.B + kChunk - 1) / kChunk;
+  RouteArgs b = a;
+  b.fuse_refine = C <= kFuseChunks ? 1 : 0;
+  const int wcnt = a.N <= kScatterMaxN ? 32 * a.N * 4 : 0;
+  const int dyn1 = kChunk * a.N * 4 + (b.fuse_refine ? wcnt : 0);
+  cudaError_t e = cudaFuncSetAttribute(score_kernel<kQ>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, dyn1);
   if (e != cudaSuccess) return e;
-  return launch_pdl(route_kernel<kMaxQ>, dim3(1), dim3(kRouteThreads), dyn, s, a);
+  e = launch_pdl(score_kernel<kQ>, dim3(C), dim3(kRouteThreads), (size_t)dyn1, s, b);
+  if (e != cudaSuccess) return e;
+  if (b.fuse_refine) {
+    if (a.events != nullptr) e = cudaEventRecord(reinterpret_cast<cudaEvent_t>(a.events[0]), s);
+    return e;
+  }
+  if (a.events != nullptr) {
+    e = cudaEventRecord(reinterpret_cast<cudaEvent_t>(a.events[0]), s);
+    if (e != cudaSuccess) return e;
+  }
+  e = cudaFuncSetAttribute(refine_kernel<kQ>, cudaFuncAttributeMaxDynamicSharedMemorySize, wcnt);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(refine_kernel<kQ>, dim3(C), dim3(kRouteThreads), (size_t)wcnt, s, b);
 }
 
 cudaError_t launch_route(const RouteArgs &a, cudaStream_t s) {
@@ -704,9 +882,10 @@ cudaError_t launch_route(const RouteArgs &a, cudaStream_t s) {
 }
 
 cudaError_t launch_router_logits(const uint16_t *x, const float *Wg, float *h, int B, int N,
-                                 int d, cudaStream_t s) {
+                                 int d, int32_t *done, cudaStream_t s) {
   dim3 grid((N + kRtExp - 1) / kRtExp, (B + kRtTok - 1) / kRtTok);
-  return launch_pdl(router_logits_kernel, grid, dim3(kRtWarps * 32), 0, s, x, Wg, h, B, N, d);
+  return launch_pdl(router_logits_kernel, grid, dim3(kRtWarps * 32), 0, s, x, Wg, h, B, N, d,
+                    done);
 }
 
 cudaError_t launch_gather(const uint16_t *x, const int32_t *perm, const Meta *meta,

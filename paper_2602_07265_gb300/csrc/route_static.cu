@@ -33,7 +33,11 @@ constexpr size_t kOffPerm = kOffOffsets + up256(sizeof(int32_t) * (kMaxN + 1));
 constexpr size_t kOffPos = kOffPerm + up256(sizeof(int32_t) * kStaticMaxPairs);
 constexpr size_t kOffTiles = kOffPos + up256(sizeof(int32_t) * kStaticMaxPairs);
 constexpr size_t kOffMeta = kOffTiles + up256(sizeof(Tile) * kStaticMaxTiles);
-constexpr size_t kStaticBytes = kOffMeta + up256(sizeof(Meta));
+constexpr int kStaticChunks = (kStaticMaxB + kChunk - 1) / kChunk;
+constexpr size_t kOffChunkCol = kOffMeta + up256(sizeof(Meta));
+constexpr size_t kOffChunkMarks = kOffChunkCol + up256(sizeof(float) * kStaticChunks * kMaxN);
+constexpr size_t kOffDone = kOffChunkMarks + up256(static_cast<size_t>(kStaticChunks) * 2 * kMaxN);
+constexpr size_t kStaticBytes = kOffDone + up256(4 * sizeof(int32_t));
 
 // The scratch itself: one copy per device that loads the library, kept until
 // the process exits.  From host code this name is only a handle for
@@ -111,8 +115,14 @@ extern "C" int xshare_route_static(const float *scores, int B, int N, int k, int
   a.counts_out = expert_counts;
   a.offsets_out = expert_offsets;
   a.perm_out = perm;
-  a.zero_words = nullptr;  // the routing kernel writes every scratch word before reading it
+  a.chunk_col = reinterpret_cast<float *>(base + kOffChunkCol);
+  a.chunk_marks = reinterpret_cast<uint8_t *>(base + kOffChunkMarks);
+  a.done = reinterpret_cast<int32_t *>(base + kOffDone);
+  a.zero_words = nullptr;
   a.zero_count = 0;
-  return launch_route(a, reinterpret_cast<cudaStream_t>(stream)) == cudaSuccess ? XS_OK
-                                                                                 : XS_ERR_CUDA;
+  // The two arrival counters must start at zero; every other scratch word is
+  // written before it is read.
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(a.done, 0, 2 * sizeof(int32_t), s) != cudaSuccess) return XS_ERR_CUDA;
+  return launch_route(a, s) == cudaSuccess ? XS_OK : XS_ERR_CUDA;
 }

@@ -43,9 +43,9 @@ constexpr int kMaxK = 16;       // top-k and warm-up k0
 constexpr int kMaxB = 8192;     // tokens
 constexpr int kTileTok = 128;   // tokens of one expert handled by one FFN tile
 constexpr int kRouteThreads = 1024;
-constexpr size_t kRouteSmemP = 96 * 1024;    // score matrix staged in shared memory up to this size
-constexpr size_t kRouteSmemIds = 64 * 1024;  // top-k ids staged in shared memory up to this size
+constexpr int kChunk = 32;                   // tokens per selection CTA (= the column-sum chunk)
 constexpr int kScatterMaxN = 256;            // parallel stable scatter up to this many experts
+constexpr int kFuseChunks = 2;               // up to this many chunks the selection CTA also refines
 
 // One FFN work tile: up to kTileTok consecutive rows of the permuted pair
 // list, all routed to `expert`.
@@ -73,6 +73,7 @@ struct Meta {
 // Byte offsets of every workspace region (256-byte aligned).
 struct Plan {
   size_t h, p, mask, ids, w, toptok, counts, offsets, perm, pos, tiles, meta;
+  size_t chunk_col, chunk_marks, done;
   size_t xp, act, out, ffn_part, ffn_cnt;
   size_t total;
   int max_pairs, max_tiles, n_sms;
@@ -98,15 +99,18 @@ struct RouteArgs {
   int32_t *counts_out;   // nullable caller copies
   int32_t *offsets_out;
   int32_t *perm_out;
+  float *chunk_col;      // [C][N] column-sum tree of each 32-token chunk
+  uint8_t *chunk_marks;  // [C][2][N] each chunk's warm-up / base marks and union marks
+  int32_t *done;         // [2] arrival counters of the two selection kernels, zero at entry
   int32_t *zero_words;   // nullable: region cleared for the FFN kernels
   int zero_count;
-  int p_smem;            // set by launch_route: scores staged in shared memory
-  int ids_smem;          // set by launch_route: ids staged in shared memory
+  void *const *events;   // nullable: events[0] is recorded between the two kernels
+  int fuse_refine;       // set by launch_route: refinement runs in the selection kernel
 };
 
 cudaError_t launch_route(const RouteArgs &a, cudaStream_t s);
 cudaError_t launch_router_logits(const uint16_t *x, const float *Wg, float *h, int B, int N,
-                                 int d, cudaStream_t s);
+                                 int d, int32_t *done, cudaStream_t s);
 cudaError_t launch_combine(const float *out, const int32_t *pos, const float *w,
                            const Meta *meta, uint16_t *y, int B, int d, int k,
                            cudaStream_t s);

@@ -73,7 +73,7 @@ def _load() -> ctypes.CDLL:
 
 LIB = _load()
 
-N_STAGES = 6
+N_STAGES = 7
 STAGE_NAMES = [LIB.xshare_stage_name(i).decode() for i in range(N_STAGES)]
 
 

@@ -35,8 +35,9 @@ def test_header_declares_the_boundary():
 
 
 def test_stage_names(X):
-    assert X.STAGE_NAMES == ["router", "select", "gather", "ffn_gate_up", "ffn_down", "combine"]
-    assert X.LIB.xshare_stage_name(6) == b""
+    assert X.STAGE_NAMES == ["router", "select", "refine", "gather", "ffn_gate_up", "ffn_down",
+                             "combine"]
+    assert X.LIB.xshare_stage_name(7) == b""
 
 
 def test_library_exports_every_declared_symbol(X):
