@@ -61,7 +61,8 @@ struct Cfg {
 struct TcParams {
   CUtensorMap tmA0;     // W_gate (gate/up) or W_down (down): [N * M, K] bf16, box 128 x 64
   CUtensorMap tmA1;     // W_up (gate/up only)
-  CUtensorMap tmB;      // xp (gate/up) or act (down): [max_pairs, K] bf16, box 16 x 64
+  CUtensorMap tmB[4];   // xp (gate/up) or act (down): [max_pairs, K] bf16, boxes of
+                        // 16, 32, 64, 128 rows x 64
   const Tile *tiles;
   Meta *meta;
   xs_stats *stats;
@@ -143,7 +144,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
     fence_mbar_init();
     prefetch_tmap(&p.tmA0);
     if (kGateUp) prefetch_tmap(&p.tmA1);
-    prefetch_tmap(&p.tmB);
+    for (int i = 0; i < 4; ++i) prefetch_tmap(&p.tmB[i]);
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), C::kTmemCols);
@@ -168,8 +169,9 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
         const int k1 = static_cast<int>(k0 + (it_end - it) < KI ? k0 + (it_end - it) : KI);
         const Tile tl = p.tiles[u / MT];
         const int mt = static_cast<int>(u % MT);
-        const int nb = (tl.ntok + kBoxTok - 1) / kBoxTok;
-        const uint32_t tx = C::kNumA * kTileBytes + nb * kBoxTok * kBK * 2;
+        // One box of 16, 32, 64 or 128 token rows covers the tile's tokens.
+        const int bsel = tl.ntok <= 16 ? 0 : tl.ntok <= 32 ? 1 : tl.ntok <= 64 ? 2 : 3;
+        const uint32_t tx = C::kNumA * kTileBytes + (kBoxTok << bsel) * kBK * 2;
         const int arow = tl.expert * p.M + mt * kBM;
         for (int kk = k0; kk < k1; ++kk) {
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, kWaitNs, abort_flag)) {
@@ -181,9 +183,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
           mbar_arrive_expect_tx(full_bar(stage), tx);
           tma_load_2d(sA, &p.tmA0, full_bar(stage), kk * kBK, arow, pol_w);
           if (kGateUp) tma_load_2d(sA + kTileBytes, &p.tmA1, full_bar(stage), kk * kBK, arow, pol_w);
-          for (int b = 0; b < nb; ++b)
-            tma_load_2d(sB + b * kBoxTok * kBK * 2, &p.tmB, full_bar(stage), kk * kBK,
-                        tl.row0 + b * kBoxTok, pol_x);
+          tma_load_2d(sB, &p.tmB[bsel], full_bar(stage), kk * kBK, tl.row0, pol_x);
           issued_mask |= 1u << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
           if (++stage == C::kStages) {
@@ -402,6 +402,13 @@ bool make_map(CUtensorMap *m, const void *base, uint64_t inner, uint64_t outer, 
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The token operand with boxes of 16, 32, 64 and 128 rows (one TMA per stage).
+bool make_token_maps(CUtensorMap (&m)[4], const void *base, uint64_t inner, uint64_t rows) {
+  for (int i = 0; i < 4; ++i)
+    if (!make_map(&m[i], base, inner, rows, static_cast<uint32_t>(kBoxTok << i))) return false;
+  return true;
+}
+
 template <bool kGateUp>
 cudaError_t launch_phase(const TcParams &p, cudaStream_t s) {
   using C = Cfg<kGateUp>;
@@ -425,7 +432,7 @@ cudaError_t launch_ffn_gate_up(const FfnArgs &a, cudaStream_t s) {
   memset(&p, 0, sizeof(p));
   if (!make_map(&p.tmA0, a.W_gate, a.d, static_cast<uint64_t>(a.N) * a.F, kBM) ||
       !make_map(&p.tmA1, a.W_up, a.d, static_cast<uint64_t>(a.N) * a.F, kBM) ||
-      !make_map(&p.tmB, a.xp, a.d, a.max_pairs, kBoxTok))
+      !make_token_maps(p.tmB, a.xp, a.d, a.max_pairs))
     return cudaErrorInvalidValue;
   p.tiles = a.tiles;
   p.meta = a.meta;
@@ -443,7 +450,7 @@ cudaError_t launch_ffn_down(const FfnArgs &a, cudaStream_t s) {
   TcParams p;
   memset(&p, 0, sizeof(p));
   if (!make_map(&p.tmA0, a.W_down, a.F, static_cast<uint64_t>(a.N) * a.d, kBM) ||
-      !make_map(&p.tmB, a.act, a.F, a.max_pairs, kBoxTok))
+      !make_token_maps(p.tmB, a.act, a.F, a.max_pairs))
     return cudaErrorInvalidValue;
   p.tmA1 = p.tmA0;
   p.tiles = a.tiles;
