@@ -361,7 +361,9 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
     barrier(world)
     e2e_ms = reduce_max(e0.elapsed_time(e1), world, dev)
 
-    launches_per_step = X.N_STAGES
+    # router, selection, [refinement: its own kernel beyond two 32-token
+    # chunks], gather, gate/up, down, combine
+    launches_per_step = X.N_STAGES - (1 if (w.B + 31) // 32 <= 2 else 0)
     out = {
         "metric": METRIC,
         "value": tokens_total / (ms_total * 1e-3),

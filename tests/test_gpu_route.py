@@ -131,6 +131,11 @@ def test_plain_topk_and_batch_on_workloads(X, name):
     (128, 64, 8, 0, W.MODE_HIER, dict(k0=0, m_r=6, tokens_per_request=64), False),   # 2 chunks/request
     (96, 64, 8, 4, W.MODE_HIER, dict(k0=2, m_r=3, tokens_per_request=32), True),
     (16, 64, 8, 0, W.MODE_HIER, dict(k0=0, m_r=3, tokens_per_request=1), False),
+    (96, 128, 8, 2, W.MODE_HIER, dict(k0=1, m_r=3, tokens_per_request=3), False),  # straddles chunks
+    (120, 128, 8, 0, W.MODE_HIER, dict(k0=1, m_r=4, tokens_per_request=8), True),  # 8 | 32
+    (144, 64, 4, 5, W.MODE_HIER, dict(k0=2, m_r=2, tokens_per_request=48), False),  # 48 > 32
+    (65, 256, 8, 24, W.MODE_BATCH, dict(k0=1), False),                          # 3 chunks, ragged
+    (64, 256, 8, 0, W.MODE_GROUP, dict(k0=1, n_groups=8, m_g=5), False),        # 2 chunks (fused)
     (256, 256, 8, 0, W.MODE_GROUP, dict(k0=0, n_groups=1, m_g=24), False),     # G = 1 is BATCH
     (256, 256, 8, 0, W.MODE_GROUP, dict(k0=1, n_groups=256, m_g=1), False),    # singleton groups
     (256, 256, 8, 0, W.MODE_GROUP, dict(k0=3, n_groups=8, m_g=2), False),      # S_0 beyond m_g G
