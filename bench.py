@@ -63,6 +63,8 @@ def parse_args(argv=None):
     ap.add_argument("--budget", type=int, default=None)
     ap.add_argument("--k0", type=int, default=None)
     ap.add_argument("--mode", default=None, choices=sorted(W.MODES))
+    ap.add_argument("--shared", type=int, default=0,
+                    help="shared experts added to every token (DeepSeek-R1 has one)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--seed", type=int, default=0)
     return ap.parse_args(argv)
@@ -86,7 +88,7 @@ def workload_from_args(args) -> W.Workload:
     return w.with_(**kw) if kw else w
 
 
-def describe(w: W.Workload) -> str:
+def describe(w: W.Workload, n_shared: int = 0) -> str:
     mode = {0: "TOPK", 1: "BATCH (Algorithm 2)", 2: "GROUP (Algorithm 6)", 3: "HIER (Algorithm 4)"}[w.mode]
     s = f"{w.name}: N={w.N} k={w.k} d={w.d} F={w.F} B={w.B} {mode}"
     if w.mode == W.MODE_BATCH:
@@ -95,6 +97,8 @@ def describe(w: W.Workload) -> str:
         s += f" m={w.budget} m_r={w.m_r} k0={w.k0} tokens/request={w.tokens_per_request}"
     elif w.mode == W.MODE_GROUP:
         s += f" G={w.n_groups} m_g={w.m_g} k0={w.k0}"
+    if n_shared:
+        s += f" + {n_shared} shared expert{'s' if n_shared > 1 else ''}"
     return s
 
 
@@ -246,15 +250,19 @@ def recorded_traffic(stage: str, units: float):
 
 # --------------------------------------------------------------------------- GPU arm
 
-def algorithmic_bytes(w: W.Workload, n_used: int, n_pairs: int) -> dict:
-    """Bytes each stage must move at least (measurement)."""
+def algorithmic_bytes(w: W.Workload, n_used: int, n_pairs: int, n_shared: int = 0) -> dict:
+    """Bytes each stage must move at least: every weight matrix it uses once,
+    plus its token rows in and out.  Shared experts count as n_shared more
+    used experts with B more rows each."""
     d, F, N, B = w.d, w.F, w.N, w.B
+    n_exp = n_used + n_shared
+    rows = n_pairs + n_shared * B
     return {
         "router": N * d * 4 + B * d * 2 + B * N * 4,
-        "ffn_gate_up": n_used * 2 * F * d * 2 + n_pairs * d * 2 + n_pairs * F * 2,
-        "ffn_down": n_used * d * F * 2 + n_pairs * F * 2 + n_pairs * d * 4,
-        "combine": n_pairs * d * 4 + B * d * 2,
-        "layer": n_used * 6 * d * F + N * d * 4 + 2 * B * d * 2,
+        "ffn_gate_up": n_exp * 2 * F * d * 2 + rows * d * 2 + rows * F * 2,
+        "ffn_down": n_exp * d * F * 2 + rows * F * 2 + rows * d * 4,
+        "combine": rows * d * 4 + B * d * 2,
+        "layer": n_exp * 6 * d * F + N * d * 4 + 2 * B * d * 2,
     }
 
 
@@ -273,8 +281,10 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
     xs_dev = [x.to(dev) for x in xs_host]
     W_g = W_g.to(dev)
     Wg, Wu, Wd = W.expert_weights(w, args.seed, device=str(dev))
+    Ns = args.shared
+    shared = W.shared_expert_weights(w, Ns, args.seed, device=str(dev)) if Ns else None
     prm = X.route_params(**w.params())
-    ws = torch.empty(X.xshare_workspace_size(w.B, w.N, w.k, w.d, w.F, w.mode, prm),
+    ws = torch.empty(X.xshare_workspace_size(w.B, w.N, w.k, w.d, w.F, w.mode, prm, Ns),
                      dtype=torch.uint8, device=dev)
     y = torch.empty(w.B, w.d, dtype=torch.bfloat16, device=dev)
     K, Wm = args.steps, args.warmup
@@ -283,7 +293,7 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
 
     def step(i, st=None, ev=None):
         X.xshare_moe_forward(xs_dev[i % N_ROTATE], W_g, Wg, Wu, Wd, w.k, w.budget, w.mode, prm,
-                             y, ws, stats=st, stage_events=ev)
+                             y, ws, stats=st, stage_events=ev, shared=shared)
 
     for i in range(Wm):
         step(i)
@@ -324,12 +334,12 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
     peaks = measured_peaks()
 
     # ---- algorithmic bytes and FLOPs ----
-    ab = [algorithmic_bytes(w, int(n_used[i]), int(n_pairs[i])) for i in range(K)]
+    ab = [algorithmic_bytes(w, int(n_used[i]), int(n_pairs[i]), Ns) for i in range(K)]
     dom_bytes = float(np.mean([a[dominant] for a in ab])) if dominant in ab[0] else None
     dom_ms = mean_ms[dominant]
     achieved = dom_bytes / (dom_ms * 1e-3) / 1e9 if dom_bytes else None
     layer_bytes = float(np.mean([a["layer"] for a in ab]))
-    flops = float(np.mean(6 * w.d * w.F * n_pairs + 2 * w.B * w.N * w.d))
+    flops = float(np.mean(6 * w.d * w.F * (n_pairs + Ns * w.B) + 2 * w.B * w.N * w.d))
     step_s = ms_total / K * 1e-3
     t_roof = max(layer_bytes / (peaks["hbm_gbs"] * 1e9), flops / (peaks["bf16_tflops"] * 1e12))
     tokens_total = reduce_sum(w.B * K, world, dev)
@@ -343,7 +353,8 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
 
     def e2e_step(i):
         x_in.copy_(x_pin[i % N_ROTATE], non_blocking=True)
-        X.xshare_moe_forward(x_in, W_g, Wg, Wu, Wd, w.k, w.budget, w.mode, prm, y, ws, stats=st_dev)
+        X.xshare_moe_forward(x_in, W_g, Wg, Wu, Wd, w.k, w.budget, w.mode, prm, y, ws, stats=st_dev,
+                             shared=shared)
         y_pin.copy_(y, non_blocking=True)
         st_pin.copy_(st_dev, non_blocking=True)
         stream.synchronize()
@@ -378,8 +389,8 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
         "dtype": "bf16",
         "data": "synthetic",
         "config": {
-            "workload": describe(w),
-            "B": w.B, "N": w.N, "k": w.k, "d": w.d, "F": w.F,
+            "workload": describe(w, Ns),
+            "B": w.B, "N": w.N, "k": w.k, "d": w.d, "F": w.F, "shared_experts": Ns,
             "global_batch": w.B * world,
             "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
             "l2": f"inputs larger than L2: ~{layer_bytes / 1e9:.2f} GB of expert weights per step "
@@ -390,7 +401,7 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
             "union_topk_mean": float(st[:, 2].mean()), "max_group_load_mean": float(st[:, 3].mean()),
         },
         "layer": {
-            "expert_weight_gbs": float(np.mean(n_used * 6 * w.d * w.F)) / step_s / 1e9,
+            "expert_weight_gbs": float(np.mean((n_used + Ns) * 6 * w.d * w.F)) / step_s / 1e9,
             "algorithmic_gbs": layer_bytes / step_s / 1e9,
             "roofline_frac": t_roof / step_s,
             "roofline_frac_vs_nominal_7900gbs": (layer_bytes / 7.9e12) / step_s,
@@ -404,7 +415,7 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
             "peak": peaks["hbm_gbs"],
             "unit": "GB/s",
             "frac": (achieved / peaks["hbm_gbs"]) if achieved else None,
-            "traffic": recorded_traffic(dominant, float(np.mean(n_used))),
+            "traffic": recorded_traffic(dominant, float(np.mean(n_used)) + Ns),
             "peak_source": f"{peaks['source']} (MEASURED_PEAKS.json hbm_gbs, copy)"
                            if peaks["source"] == "measured" else "fallback 6.8 TB/s",
         },
@@ -431,9 +442,10 @@ class OracleSampler:
     F / f_rows.  Inputs and the needed expert weights are prepared once,
     outside the timed calls."""
 
-    def __init__(self, w: W.Workload, seed: int, ffn_tokens: int, f_rows: int):
+    def __init__(self, w: W.Workload, seed: int, ffn_tokens: int, f_rows: int,
+                 n_shared: int = 0):
         from oracle import xshare_oracle as O
-        self.O, self.w = O, w
+        self.O, self.w, self.n_shared = O, w, n_shared
         self.f_rows = min(f_rows, w.F)
         x, W_g = W.router_inputs(w, seed)
         self.xb, self.W_g = W.bf16_bits(x), W_g.numpy()
@@ -447,6 +459,12 @@ class OracleSampler:
                                           f_rows=self.f_rows)
             for i, e in enumerate(self.experts):
                 self.weights[e] = (W.bf16_bits(Wg[i]), W.bf16_bits(Wu[i]), W.bf16_bits(Wd[i]))
+        self.shared = []
+        if n_shared:
+            Sg, Su, Sd = W.expert_weights(w.with_(N=n_shared), seed + 7_777_777, device="cpu",
+                                          f_rows=self.f_rows)
+            self.shared = [(W.bf16_bits(Sg[j]), W.bf16_bits(Su[j]), W.bf16_bits(Sd[j]))
+                           for j in range(n_shared)]
 
     def step(self) -> dict:
         O, w = self.O, self.w
@@ -458,17 +476,20 @@ class OracleSampler:
         t1 = time.perf_counter()
         if self.tokens:
             O.moe_ffn_combine(self.xb, r["ids"], r["w"], self.weights.__getitem__, tokens=self.tokens)
+            if self.n_shared:
+                O.shared_experts_out(self.xb, self.shared.__getitem__, self.n_shared, self.tokens)
         t_ffn = (time.perf_counter() - t1) * (w.F / self.f_rows)
         per_token = t_route / w.B + (t_ffn / len(self.tokens) if self.tokens else 0.0)
         return {"t_route": t_route, "t_ffn_scaled": t_ffn, "per_token_s": per_token}
 
     def describe(self, s: dict) -> str:
-        return (f"full selection of one {self.w.B}-token batch ({s['t_route']:.2f} s) + expert FFN "
+        sh = f" (+ {self.n_shared} shared)" if self.n_shared else ""
+        return (f"full selection of one {self.w.B}-token batch ({s['t_route']:.2f} s) + expert FFN{sh} "
                 f"and combine of {len(self.tokens)} token(s) on {self.f_rows}/{self.w.F} hidden units, "
                 f"scaled to F ({s['t_ffn_scaled']:.2f} s); numpy fp64, 1 thread")
 
 
-def cpu_baseline(w: W.Workload, seed: int) -> dict:
+def cpu_baseline(w: W.Workload, seed: int, n_shared: int = 0) -> dict:
     """The oracle, single-threaded, on a bounded sample, in a child process so
     that BLAS is pinned to one thread."""
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
@@ -478,7 +499,7 @@ def cpu_baseline(w: W.Workload, seed: int) -> dict:
     code = (f"import sys, json; sys.path.insert(0, {ROOT!r}); import torch; torch.set_num_threads(1); "
             f"import bench; from paper_2602_07265_gb300 import workloads as W; "
             f"w = W.WORKLOADS[{w.name!r}].with_(**{kw}); "
-            f"o = bench.OracleSampler(w, {seed}, 4, {f_rows}); o.step(); s = o.step(); "
+            f"o = bench.OracleSampler(w, {seed}, 4, {f_rows}, {int(n_shared)}); o.step(); s = o.step(); "
             f"s['describe'] = o.describe(s); print(json.dumps(s))")
     r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
                        timeout=900)
@@ -497,7 +518,7 @@ def run_reference(args, w: W.Workload, rank: int, world: int) -> dict:
     Steps beyond a ~150 s budget are skipped, keeping at least 3."""
     torch.set_num_threads(1)
     K, Wm = args.steps, args.warmup
-    sampler = OracleSampler(w, args.seed, 1, max(128, w.F // 8))
+    sampler = OracleSampler(w, args.seed, 1, max(128, w.F // 8), args.shared)
     for _ in range(min(Wm, 3)):
         s = sampler.step()
     budget_s, spent, per_token = 150.0, 0.0, []
@@ -515,8 +536,8 @@ def run_reference(args, w: W.Workload, rank: int, world: int) -> dict:
         "warmup": Wm, "ms_per_step": 1e3 * w.B / value, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "impl": "reference",
-        "config": {"workload": describe(w), "B": w.B, "N": w.N, "k": w.k, "d": w.d, "F": w.F,
-                   "global_batch": w.B, "parallelism": "cpu oracle, rank 0 only"},
+        "config": {"workload": describe(w, args.shared), "B": w.B, "N": w.N, "k": w.k, "d": w.d,
+                   "F": w.F, "shared_experts": args.shared, "global_batch": w.B, "parallelism": "cpu oracle, rank 0 only"},
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
@@ -538,7 +559,7 @@ def main(argv=None):
     out = run_gpu(args, w, rank, world, local)
     if rank == 0:
         if world == 1 and not args.no_cpu_baseline:
-            out["cpu_baseline"] = cpu_baseline(w, args.seed)
+            out["cpu_baseline"] = cpu_baseline(w, args.seed, args.shared)
         print(json.dumps(out))
     if world > 1:
         torch.distributed.destroy_process_group()

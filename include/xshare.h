@@ -101,11 +101,22 @@ typedef struct {
 #define XS_DEV_OK 0
 #define XS_DEV_TIMEOUT 1      /* a bounded wait inside a kernel ran out */
 
+/* Shared experts E^s_j of the layer (Sec. 2.1: y = sum_i g_i E_i(x) +
+ * sum_j E^s_j(x)): every token goes through each of them with weight 1.
+ * Same shapes per expert as the routed ones (d_ff = F), device pointers:
+ * W_gate, W_up [n_shared, F, d] bf16; W_down [n_shared, d, F] bf16. */
+typedef struct {
+  const uint16_t *W_gate;
+  const uint16_t *W_up;
+  const uint16_t *W_down;
+  int32_t n_shared;           /* 0 .. 8 */
+} xs_shared_experts;
+
 /* Bytes of workspace the calls below need for these sizes.  For
- * xshare_route pass d = F = 0.  Returns 0 for arguments the calls would
- * reject.  Depends on the current device's SM count. */
+ * xshare_route pass d = F = 0 and n_shared = 0.  Returns 0 for arguments the
+ * calls would reject.  Depends on the current device's SM count. */
 size_t xshare_workspace_size(int B, int N, int k, int d, int F, int mode,
-                             const xs_route_params *prm);
+                             const xs_route_params *prm, int n_shared);
 
 /* Steps a3-a7 of the path: batch-aware selection and refinement on given scores.
  *
@@ -133,25 +144,28 @@ int xshare_route(const float *scores, int B, int N, int k, int budget, int mode,
                  int32_t *expert_offsets, int32_t *perm, void *workspace,
                  size_t ws_bytes, xs_stream_t stream);
 
-/* The whole path a1-a9: one MoE layer forward, routed part (Sec. 2.1).
+/* The whole path a1-a9: one MoE layer forward (Sec. 2.1).
  *
  *   x       [B, d] bf16, device: token hidden states.
  *   W_g     [N, d] fp32, device: router weights; h = W_g x (Sec. 2.2).
  *   W_gate  [N, F, d] bf16, device; W_up [N, F, d] bf16; W_down [N, d, F] bf16:
  *           expert e computes E_e(x) = W_down[e] (silu(W_gate[e] x) * (W_up[e] x)).
  *           Only the experts that receive a token are read.
- *   y       [B, d] bf16, device, out: y_t = sum over slots of w_ts E_{ids_ts}(x_t),
- *           accumulated in fp32 and rounded once to bf16.
+ *   shared  nullable: shared experts, added to every token's output.
+ *   y       [B, d] bf16, device, out: y_t = sum over slots of w_ts E_{ids_ts}(x_t)
+ *           + sum_j E^s_j(x_t), accumulated in fp32 (routed slots in slot order,
+ *           then the shared experts in order) and rounded once to bf16.
  *   scores_out [B, N] fp32, device, out, nullable: the dense softmax scores g.
  *   sel_mask, topk_ids, topk_w, stats: as in xshare_route, each nullable.
- * Other arguments as in xshare_route.
+ * Other arguments as in xshare_route; the workspace size is
+ * xshare_workspace_size(B, N, k, d, F, mode, prm, shared ? shared->n_shared : 0).
  */
 int xshare_moe_forward(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
                        const uint16_t *W_up, const uint16_t *W_down, int B, int d, int F,
                        int N, int k, int budget, int mode, const xs_route_params *prm,
-                       uint16_t *y, float *scores_out, uint8_t *sel_mask,
-                       int32_t *topk_ids, float *topk_w, xs_stats *stats, void *workspace,
-                       size_t ws_bytes, xs_stream_t stream);
+                       const xs_shared_experts *shared, uint16_t *y, float *scores_out,
+                       uint8_t *sel_mask, int32_t *topk_ids, float *topk_w, xs_stats *stats,
+                       void *workspace, size_t ws_bytes, xs_stream_t stream);
 
 /* xshare_route for callers that cannot allocate device memory.  The paper has
  * no counterpart: this is a deployment convenience of the library.
@@ -194,10 +208,11 @@ int xshare_route_static(const float *scores, int B, int N, int k, int budget, in
 int xshare_moe_forward_profiled(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
                                 const uint16_t *W_up, const uint16_t *W_down, int B, int d,
                                 int F, int N, int k, int budget, int mode,
-                                const xs_route_params *prm, uint16_t *y, float *scores_out,
-                                uint8_t *sel_mask, int32_t *topk_ids, float *topk_w,
-                                xs_stats *stats, void *workspace, size_t ws_bytes,
-                                xs_stream_t stream, void *const *stage_events);
+                                const xs_route_params *prm, const xs_shared_experts *shared,
+                                uint16_t *y, float *scores_out, uint8_t *sel_mask,
+                                int32_t *topk_ids, float *topk_w, xs_stats *stats,
+                                void *workspace, size_t ws_bytes, xs_stream_t stream,
+                                void *const *stage_events);
 
 /* Name of stage i of xshare_moe_forward (e.g. "router"), or "" if out of range. */
 const char *xshare_stage_name(int i);

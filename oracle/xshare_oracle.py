@@ -441,20 +441,41 @@ def moe_ffn_combine(x_bits: np.ndarray, ids: np.ndarray, w: np.ndarray,
     return combine(ids, w, out, tokens, d)
 
 
+def shared_experts_out(x_bits: np.ndarray, get_shared, n_shared: int,
+                       tokens: Sequence[int]) -> np.ndarray:
+    """Sum over the shared experts of E^s_j(x_t) (Sec. 2.1, second term), fp64.
+
+    get_shared(j) -> (Wgate [F, d], Wup [F, d], Wdown [d, F]) uint16 bf16 patterns.
+    """
+    x = bf16_bits_to_f64(x_bits)[list(tokens)]
+    out = np.zeros((len(tokens), x.shape[1]), dtype=np.float64)
+    for j in range(n_shared):
+        Wg, Wu, Wd = get_shared(j)
+        out += expert_ffn(x, Wg, Wu, Wd)
+    return out
+
+
 def moe_forward(x_bits: np.ndarray, W_g: np.ndarray, get_expert, k: int, budget: int,
-                mode: int, tokens: Optional[Sequence[int]] = None, **params) -> Dict[str, object]:
+                mode: int, tokens: Optional[Sequence[int]] = None, get_shared=None,
+                n_shared: int = 0, **params) -> Dict[str, object]:
     """One MoE layer forward: router, dense softmax, selection, refinement,
-    permutation, expert FFN over the routed pairs and weighted combine.
+    permutation, expert FFN over the routed pairs and weighted combine, plus
+    the shared experts when given (Sec. 2.1):
+        y = sum_i g_i(x) E_i(x) + sum_j E^s_j(x).
 
     Returns the routing dictionary of `route` plus "h" (fp64 logits), "p" (fp32
-    scores) and "y" (fp64 routed output for `tokens`, all by default).
+    scores) and "y" (fp64 output for `tokens`, all by default).
     """
     h = router_logits(x_bits, W_g)
     p = softmax_scores(h)
     r = route(p, k, budget, mode, **params)
     r["h"] = h
     r["p"] = p
-    r["y"] = moe_ffn_combine(x_bits, r["ids"], r["w"], get_expert, tokens)
+    toks = list(range(x_bits.shape[0])) if tokens is None else list(tokens)
+    y = moe_ffn_combine(x_bits, r["ids"], r["w"], get_expert, toks)
+    if n_shared:
+        y = y + shared_experts_out(x_bits, get_shared, n_shared, toks)
+    r["y"] = y
     return r
 
 

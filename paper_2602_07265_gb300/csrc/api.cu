@@ -100,12 +100,13 @@ RouteArgs route_args(const Plan &pl, void *ws, int B, int N, int k, int budget, 
 
 }  // namespace
 
-Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms) {
+Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms, int n_shared) {
   Plan pl;
   std::memset(&pl, 0, sizeof(pl));
   pl.n_sms = n_sms;
   pl.max_pairs = B * k;
-  pl.max_tiles = N + (B * k) / kTileTok + 1;
+  pl.max_rows = B * k + n_shared * B;
+  pl.max_tiles = N + (B * k) / kTileTok + 1 + n_shared * ((B + kTileTok - 1) / kTileTok);
   size_t o = 0;
   auto take = [&](size_t bytes) {
     size_t r = o;
@@ -129,9 +130,9 @@ Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms) {
   pl.chunk_marks = take((size_t)chunks * 2 * N);
   pl.done = take(4 * sizeof(int32_t));
   if (with_ffn) {
-    pl.xp = take((size_t)pl.max_pairs * d * 2);
-    pl.act = take((size_t)pl.max_pairs * F * 2);
-    pl.out = take((size_t)pl.max_pairs * d * 4);
+    pl.xp = take((size_t)pl.max_rows * d * 2);
+    pl.act = take((size_t)pl.max_rows * F * 2);
+    pl.out = take((size_t)pl.max_rows * d * 4);
     pl.ffn_part = take(ffn_part_bytes(n_sms));
     pl.ffn_cnt = take(ffn_cnt_words(pl.max_tiles, B, d, F) * 4);
   }
@@ -144,13 +145,14 @@ Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms) {
 using namespace xs;
 
 extern "C" size_t xshare_workspace_size(int B, int N, int k, int d, int F, int mode,
-                                        const xs_route_params *prm) {
+                                        const xs_route_params *prm, int n_shared) {
   if (check_route_args(B, N, k, 0, mode, prm) != XS_OK) return 0;
   const bool ffn = (d != 0 || F != 0);
   if (ffn && check_ffn_shape(d, F) != XS_OK) return 0;
+  if (n_shared < 0 || n_shared > kMaxShared || (!ffn && n_shared != 0)) return 0;
   const int sms = current_device_sms();
   if (sms < 0) return 0;
-  return make_plan(B, N, k, d, F, ffn, sms).total;
+  return make_plan(B, N, k, d, F, ffn, sms, n_shared).total;
 }
 
 extern "C" int xshare_route(const float *scores, int B, int N, int k, int budget, int mode,
@@ -165,7 +167,7 @@ extern "C" int xshare_route(const float *scores, int B, int N, int k, int budget
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return XS_ERR_WORKSPACE;
   const int sms = current_device_sms();
   if (sms < 0) return sms;
-  const Plan pl = make_plan(B, N, k, 0, 0, false, sms);
+  const Plan pl = make_plan(B, N, k, 0, 0, false, sms, 0);
   if (ws_bytes < pl.total) return XS_ERR_WORKSPACE;
   RouteArgs a = route_args(pl, workspace, B, N, k, budget, mode, prm);
   a.p = const_cast<float *>(scores);  // read only when logits == nullptr
@@ -188,10 +190,10 @@ const char *const kStageNames[XS_N_STAGES] = {"router", "select", "refine", "gat
 
 int forward_impl(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
                  const uint16_t *W_up, const uint16_t *W_down, int B, int d, int F, int N, int k,
-                 int budget, int mode, const xs_route_params *prm, uint16_t *y,
-                 float *scores_out, uint8_t *sel_mask, int32_t *topk_ids, float *topk_w,
-                 xs_stats *stats, void *workspace, size_t ws_bytes, xs_stream_t stream,
-                 void *const *events) {
+                 int budget, int mode, const xs_route_params *prm,
+                 const xs_shared_experts *shared, uint16_t *y, float *scores_out,
+                 uint8_t *sel_mask, int32_t *topk_ids, float *topk_w, xs_stats *stats,
+                 void *workspace, size_t ws_bytes, xs_stream_t stream, void *const *events) {
   int rc = check_route_args(B, N, k, budget, mode, prm);
   if (rc != XS_OK) return rc;
   rc = check_ffn_shape(d, F);
@@ -200,10 +202,17 @@ int forward_impl(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
   if (!aligned16(x) || !aligned16(W_g) || !aligned16(W_gate) || !aligned16(W_up) ||
       !aligned16(W_down) || !aligned16(y) || (scores_out && !aligned16(scores_out)))
     return XS_ERR_ALIGN;
+  const int n_shared = shared ? shared->n_shared : 0;
+  if (n_shared < 0 || n_shared > kMaxShared) return XS_ERR_PARAM;
+  if (n_shared > 0) {
+    if (!shared->W_gate || !shared->W_up || !shared->W_down) return XS_ERR_NULL;
+    if (!aligned16(shared->W_gate) || !aligned16(shared->W_up) || !aligned16(shared->W_down))
+      return XS_ERR_ALIGN;
+  }
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return XS_ERR_WORKSPACE;
   const int sms = current_device_sms();
   if (sms < 0) return sms;
-  const Plan pl = make_plan(B, N, k, d, F, true, sms);
+  const Plan pl = make_plan(B, N, k, d, F, true, sms, n_shared);
   if (ws_bytes < pl.total) return XS_ERR_WORKSPACE;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
@@ -217,12 +226,19 @@ int forward_impl(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
   a.stats = stats;
   a.zero_words = at<int32_t>(workspace, pl.ffn_cnt);
   a.zero_count = (int)ffn_cnt_words(pl.max_tiles, B, d, F);
+  a.n_shared = n_shared;
 
   FfnArgs f;
   std::memset(&f, 0, sizeof(f));
   f.W_gate = W_gate;
   f.W_up = W_up;
   f.W_down = W_down;
+  if (n_shared > 0) {
+    f.S_gate = shared->W_gate;
+    f.S_up = shared->W_up;
+    f.S_down = shared->W_down;
+  }
+  f.n_shared = n_shared;
   f.xp = at<uint16_t>(workspace, pl.xp);
   f.act = at<uint16_t>(workspace, pl.act);
   f.out = at<float>(workspace, pl.out);
@@ -234,7 +250,7 @@ int forward_impl(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
   f.N = N;
   f.d = d;
   f.F = F;
-  f.max_pairs = pl.max_pairs;
+  f.max_rows = pl.max_rows;
   f.max_tiles = pl.max_tiles;
   f.n_sms = sms;
 
@@ -247,13 +263,14 @@ int forward_impl(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
     return XS_ERR_CUDA;
   a.events = events ? events + 2 : nullptr;  // between the selection and refinement kernels
   if (launch_route(a, s) != cudaSuccess || !mark(3)) return XS_ERR_CUDA;
-  if (launch_gather(x, a.perm, a.meta, const_cast<uint16_t *>(f.xp), pl.max_pairs, d, k, s) !=
+  if (launch_gather(x, a.perm, a.meta, const_cast<uint16_t *>(f.xp), pl.max_rows, B, d, k, s) !=
           cudaSuccess ||
       !mark(4))
     return XS_ERR_CUDA;
   if (launch_ffn_gate_up(f, s) != cudaSuccess || !mark(5)) return XS_ERR_CUDA;
   if (launch_ffn_down(f, s) != cudaSuccess || !mark(6)) return XS_ERR_CUDA;
-  if (launch_combine(f.out, a.pos, a.w, a.meta, y, B, d, k, s) != cudaSuccess || !mark(7))
+  if (launch_combine(f.out, a.pos, a.w, a.meta, y, B, d, k, n_shared, s) != cudaSuccess ||
+      !mark(7))
     return XS_ERR_CUDA;
   return XS_OK;
 }
@@ -263,11 +280,11 @@ int forward_impl(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
 extern "C" int xshare_moe_forward(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
                                   const uint16_t *W_up, const uint16_t *W_down, int B, int d,
                                   int F, int N, int k, int budget, int mode,
-                                  const xs_route_params *prm, uint16_t *y, float *scores_out,
-                                  uint8_t *sel_mask, int32_t *topk_ids, float *topk_w,
-                                  xs_stats *stats, void *workspace, size_t ws_bytes,
-                                  xs_stream_t stream) {
-  return forward_impl(x, W_g, W_gate, W_up, W_down, B, d, F, N, k, budget, mode, prm, y,
+                                  const xs_route_params *prm, const xs_shared_experts *shared,
+                                  uint16_t *y, float *scores_out, uint8_t *sel_mask,
+                                  int32_t *topk_ids, float *topk_w, xs_stats *stats,
+                                  void *workspace, size_t ws_bytes, xs_stream_t stream) {
+  return forward_impl(x, W_g, W_gate, W_up, W_down, B, d, F, N, k, budget, mode, prm, shared, y,
                       scores_out, sel_mask, topk_ids, topk_w, stats, workspace, ws_bytes, stream,
                       nullptr);
 }
@@ -276,7 +293,8 @@ extern "C" int xshare_moe_forward_profiled(const uint16_t *x, const float *W_g,
                                            const uint16_t *W_gate, const uint16_t *W_up,
                                            const uint16_t *W_down, int B, int d, int F, int N,
                                            int k, int budget, int mode,
-                                           const xs_route_params *prm, uint16_t *y,
+                                           const xs_route_params *prm,
+                                           const xs_shared_experts *shared, uint16_t *y,
                                            float *scores_out, uint8_t *sel_mask,
                                            int32_t *topk_ids, float *topk_w, xs_stats *stats,
                                            void *workspace, size_t ws_bytes, xs_stream_t stream,
@@ -284,7 +302,7 @@ extern "C" int xshare_moe_forward_profiled(const uint16_t *x, const float *W_g,
   if (stage_events == nullptr) return XS_ERR_NULL;
   for (int i = 0; i <= XS_N_STAGES; ++i)
     if (stage_events[i] == nullptr) return XS_ERR_NULL;
-  return forward_impl(x, W_g, W_gate, W_up, W_down, B, d, F, N, k, budget, mode, prm, y,
+  return forward_impl(x, W_g, W_gate, W_up, W_down, B, d, F, N, k, budget, mode, prm, shared, y,
                       scores_out, sel_mask, topk_ids, topk_w, stats, workspace, ws_bytes, stream,
                       stage_events);
 }

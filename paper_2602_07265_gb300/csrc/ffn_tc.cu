@@ -61,18 +61,22 @@ struct Cfg {
 struct TcParams {
   CUtensorMap tmA0;     // W_gate (gate/up) or W_down (down): [N * M, K] bf16, box 128 x 64
   CUtensorMap tmA1;     // W_up (gate/up only)
-  CUtensorMap tmB[4];   // xp (gate/up) or act (down): [max_pairs, K] bf16, boxes of
+  CUtensorMap tmS0;     // the same for the shared experts (experts >= n_routed)
+  CUtensorMap tmS1;
+  CUtensorMap tmB[4];   // xp (gate/up) or act (down): [max_rows, K] bf16, boxes of
                         // 16, 32, 64, 128 rows x 64
   const Tile *tiles;
   Meta *meta;
   xs_stats *stats;
   float *part;          // [grid][2 slots][kNumA][128 cols][128 lanes] fp32
   int32_t *cnt;         // [units] arrival counters, zeroed by the routing kernel
-  uint16_t *act_out;    // gate/up output [max_pairs, M]
-  float *out;           // down output [max_pairs, M]
+  uint16_t *act_out;    // gate/up output [max_rows, M]
+  float *out;           // down output [max_rows, M]
   int M;                // weight rows per expert: F (gate/up) or d (down)
   int K;                // reduction length: d (gate/up) or F (down)
   int grid;
+  int n_routed;         // N: tiles of experts >= N use tmS0 / tmS1
+  int has_shared;
 };
 
 struct Range {
@@ -144,6 +148,10 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
     fence_mbar_init();
     prefetch_tmap(&p.tmA0);
     if (kGateUp) prefetch_tmap(&p.tmA1);
+    if (p.has_shared) {
+      prefetch_tmap(&p.tmS0);
+      if (kGateUp) prefetch_tmap(&p.tmS1);
+    }
     for (int i = 0; i < 4; ++i) prefetch_tmap(&p.tmB[i]);
   }
   if (warp == 1) {
@@ -172,7 +180,10 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
         // One box of 16, 32, 64 or 128 token rows covers the tile's tokens.
         const int bsel = tl.ntok <= 16 ? 0 : tl.ntok <= 32 ? 1 : tl.ntok <= 64 ? 2 : 3;
         const uint32_t tx = C::kNumA * kTileBytes + (kBoxTok << bsel) * kBK * 2;
-        const int arow = tl.expert * p.M + mt * kBM;
+        const bool routed = tl.expert < p.n_routed;
+        const CUtensorMap *mA0 = routed ? &p.tmA0 : &p.tmS0;
+        const CUtensorMap *mA1 = routed ? &p.tmA1 : &p.tmS1;
+        const int arow = (routed ? tl.expert : tl.expert - p.n_routed) * p.M + mt * kBM;
         for (int kk = k0; kk < k1; ++kk) {
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, kWaitNs, abort_flag)) {
             ok = false;
@@ -181,8 +192,8 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
           const uint32_t sA = sbase + stage * C::kStageBytes;
           const uint32_t sB = sA + C::kNumA * kTileBytes;
           mbar_arrive_expect_tx(full_bar(stage), tx);
-          tma_load_2d(sA, &p.tmA0, full_bar(stage), kk * kBK, arow, pol_w);
-          if (kGateUp) tma_load_2d(sA + kTileBytes, &p.tmA1, full_bar(stage), kk * kBK, arow, pol_w);
+          tma_load_2d(sA, mA0, full_bar(stage), kk * kBK, arow, pol_w);
+          if (kGateUp) tma_load_2d(sA + kTileBytes, mA1, full_bar(stage), kk * kBK, arow, pol_w);
           tma_load_2d(sB, &p.tmB[bsel], full_bar(stage), kk * kBK, tl.row0, pol_x);
           issued_mask |= 1u << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
@@ -432,8 +443,18 @@ cudaError_t launch_ffn_gate_up(const FfnArgs &a, cudaStream_t s) {
   memset(&p, 0, sizeof(p));
   if (!make_map(&p.tmA0, a.W_gate, a.d, static_cast<uint64_t>(a.N) * a.F, kBM) ||
       !make_map(&p.tmA1, a.W_up, a.d, static_cast<uint64_t>(a.N) * a.F, kBM) ||
-      !make_token_maps(p.tmB, a.xp, a.d, a.max_pairs))
+      !make_token_maps(p.tmB, a.xp, a.d, a.max_rows))
     return cudaErrorInvalidValue;
+  if (a.n_shared > 0) {
+    if (!make_map(&p.tmS0, a.S_gate, a.d, static_cast<uint64_t>(a.n_shared) * a.F, kBM) ||
+        !make_map(&p.tmS1, a.S_up, a.d, static_cast<uint64_t>(a.n_shared) * a.F, kBM))
+      return cudaErrorInvalidValue;
+  } else {
+    p.tmS0 = p.tmA0;
+    p.tmS1 = p.tmA1;
+  }
+  p.n_routed = a.N;
+  p.has_shared = a.n_shared > 0;
   p.tiles = a.tiles;
   p.meta = a.meta;
   p.stats = a.stats;
@@ -450,9 +471,18 @@ cudaError_t launch_ffn_down(const FfnArgs &a, cudaStream_t s) {
   TcParams p;
   memset(&p, 0, sizeof(p));
   if (!make_map(&p.tmA0, a.W_down, a.F, static_cast<uint64_t>(a.N) * a.d, kBM) ||
-      !make_token_maps(p.tmB, a.act, a.F, a.max_pairs))
+      !make_token_maps(p.tmB, a.act, a.F, a.max_rows))
     return cudaErrorInvalidValue;
   p.tmA1 = p.tmA0;
+  if (a.n_shared > 0) {
+    if (!make_map(&p.tmS0, a.S_down, a.F, static_cast<uint64_t>(a.n_shared) * a.d, kBM))
+      return cudaErrorInvalidValue;
+  } else {
+    p.tmS0 = p.tmA0;
+  }
+  p.tmS1 = p.tmS0;
+  p.n_routed = a.N;
+  p.has_shared = a.n_shared > 0;
   p.tiles = a.tiles;
   p.meta = a.meta;
   p.stats = a.stats;

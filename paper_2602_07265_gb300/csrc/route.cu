@@ -295,6 +295,17 @@ __device__ void build_permutation(const RouteArgs &a, PermSmem sm) {
       sm.scal[2] = tot[1];  // tiles
       sm.scal[3] = tot[2];  // used experts
     }
+    // Shared experts: every token, in token order, after the routed pairs.
+    const int tpt = (B + kTileTok - 1) / kTileTok;
+    for (int i = tid; i < a.n_shared * tpt; i += blockDim.x) {
+      const int j = i / tpt, tt = i - j * tpt;
+      Tile tl;
+      tl.expert = N + j;
+      tl.row0 = tot[0] + j * B + tt * kTileTok;
+      tl.ntok = min(kTileTok, B - tt * kTileTok);
+      tl.pad = 0;
+      a.tiles[tot[1] + i] = tl;
+    }
   }
   __syncthreads();
   const unsigned lt = (1u << lane) - 1u;
@@ -357,8 +368,9 @@ __device__ void build_permutation(const RouteArgs &a, PermSmem sm) {
   if (tid == 0) {
     Meta m = *a.meta;
     m.n_pairs = sm.scal[1];  // == B * kp unless scores were non-finite
-    m.n_tiles = sm.scal[2];
+    m.n_tiles = sm.scal[2] + a.n_shared * ((B + kTileTok - 1) / kTileTok);
     m.n_used = sm.scal[3];
+    m.n_rows = sm.scal[1] + a.n_shared * B;
     *a.meta = m;
     if (a.stats) {
       xs_stats st;
@@ -645,9 +657,10 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   for (int j = tid; j < N; j += blockDim.x) a.mask[j] = s_mask[j];
   if (tid == 0) {
     Meta m;
-    for (int i = 0; i < 8; ++i) m.pad[i] = 0;
+    for (int i = 0; i < 7; ++i) m.pad[i] = 0;
     m.n_pairs = 0;
     m.n_tiles = 0;
+    m.n_rows = 0;
     m.kprime = min(k, nsel);
     m.n_selected = nsel;
     m.n_used = 0;
@@ -805,23 +818,27 @@ __global__ void __launch_bounds__(kRtWarps * 32) router_logits_kernel(
 __global__ void __launch_bounds__(256) gather_kernel(const uint16_t *__restrict__ x,
                                                      const int32_t *__restrict__ perm,
                                                      const Meta *__restrict__ meta,
-                                                     uint16_t *__restrict__ xp, int d, int k) {
+                                                     uint16_t *__restrict__ xp, int B, int d,
+                                                     int k) {
   pdl_wait();
   pdl_trigger();
   const int row = blockIdx.x;
-  if (row >= meta->n_pairs) return;
-  const int t = perm[row] / k;
+  const int P = meta->n_pairs;
+  if (row >= meta->n_rows) return;
+  const int t = row < P ? perm[row] / k : (row - P) % B;  // routed pair, else shared row
   const uint4 *src = reinterpret_cast<const uint4 *>(x + (size_t)t * d);
   uint4 *dst = reinterpret_cast<uint4 *>(xp + (size_t)row * d);
   for (int i = threadIdx.x; i < d / 8; i += blockDim.x) dst[i] = __ldg(src + i);
 }
 
-// ---- a9: y_t = sum over slots s < k' of w_ts * out[pos(t, s)], fp32, bf16 once.
+// ---- a9: y_t = sum over slots s < k' of w_ts * out[pos(t, s)]
+//              + sum over shared experts j of out[n_pairs + j * B + t], fp32, bf16 once.
 __global__ void __launch_bounds__(256) combine_kernel(const float *__restrict__ out,
                                                       const int32_t *__restrict__ pos,
                                                       const float *__restrict__ w,
                                                       const Meta *__restrict__ meta,
-                                                      uint16_t *__restrict__ y, int d, int k) {
+                                                      uint16_t *__restrict__ y, int B, int d,
+                                                      int k, int n_shared) {
   pdl_wait();
   pdl_trigger();
   const int t = blockIdx.y;
@@ -838,6 +855,14 @@ __global__ void __launch_bounds__(256) combine_kernel(const float *__restrict__ 
     acc.y = fmaf(ws, o.y, acc.y);
     acc.z = fmaf(ws, o.z, acc.z);
     acc.w = fmaf(ws, o.w, acc.w);
+  }
+  for (int j = 0; j < n_shared; ++j) {
+    const size_t r = (size_t)meta->n_pairs + (size_t)j * B + t;
+    const float4 o = reinterpret_cast<const float4 *>(out + r * d)[c4];
+    acc.x += o.x;
+    acc.y += o.y;
+    acc.z += o.z;
+    acc.w += o.w;
   }
   __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x, acc.y);
   __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z, acc.w);
@@ -889,15 +914,16 @@ cudaError_t launch_router_logits(const uint16_t *x, const float *Wg, float *h, i
 }
 
 cudaError_t launch_gather(const uint16_t *x, const int32_t *perm, const Meta *meta,
-                          uint16_t *xp, int max_pairs, int d, int k, cudaStream_t s) {
-  return launch_pdl(gather_kernel, dim3(max_pairs), dim3(256), 0, s, x, perm, meta, xp, d, k);
+                          uint16_t *xp, int max_rows, int B, int d, int k, cudaStream_t s) {
+  return launch_pdl(gather_kernel, dim3(max_rows), dim3(256), 0, s, x, perm, meta, xp, B, d, k);
 }
 
 cudaError_t launch_combine(const float *out, const int32_t *pos, const float *w,
-                           const Meta *meta, uint16_t *y, int B, int d, int k,
+                           const Meta *meta, uint16_t *y, int B, int d, int k, int n_shared,
                            cudaStream_t s) {
   dim3 grid((d / 4 + 255) / 256, B);
-  return launch_pdl(combine_kernel, grid, dim3(256), 0, s, out, pos, w, meta, y, d, k);
+  return launch_pdl(combine_kernel, grid, dim3(256), 0, s, out, pos, w, meta, y, B, d, k,
+                    n_shared);
 }
 
 }  // namespace xs

@@ -46,9 +46,12 @@ constexpr int kRouteThreads = 1024;
 constexpr int kChunk = 32;                   // tokens per selection CTA (= the column-sum chunk)
 constexpr int kScatterMaxN = 256;            // parallel stable scatter up to this many experts
 constexpr int kFuseChunks = 2;               // up to this many chunks the selection CTA also refines
+constexpr int kMaxShared = 8;                // shared experts
 
 // One FFN work tile: up to kTileTok consecutive rows of the permuted pair
-// list, all routed to `expert`.
+// list, all routed to `expert`.  Experts N .. N + n_shared - 1 are the shared
+// experts; their rows follow the routed pairs: row n_pairs + j * B + t is
+// token t's pass through shared expert j.
 struct Tile {
   int32_t expert;
   int32_t row0;
@@ -67,7 +70,8 @@ struct Meta {
   int32_t union_topk;
   int32_t max_group_load;
   int32_t status;       // XS_DEV_*
-  int32_t pad[8];
+  int32_t n_rows;       // FFN rows: n_pairs + n_shared * B
+  int32_t pad[7];
 };
 
 // Byte offsets of every workspace region (256-byte aligned).
@@ -76,10 +80,12 @@ struct Plan {
   size_t chunk_col, chunk_marks, done;
   size_t xp, act, out, ffn_part, ffn_cnt;
   size_t total;
-  int max_pairs, max_tiles, n_sms;
+  int max_pairs;   // routed pairs B * k
+  int max_rows;    // FFN rows: routed pairs plus n_shared * B
+  int max_tiles, n_sms;
 };
 
-Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms);
+Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms, int n_shared);
 
 struct RouteArgs {
   const float *logits;   // nullable: if set, p = softmax(logits) is computed first
@@ -106,28 +112,31 @@ struct RouteArgs {
   int zero_count;
   void *const *events;   // nullable: events[0] is recorded between the two kernels
   int fuse_refine;       // set by launch_route: refinement runs in the selection kernel
+  int n_shared;          // shared-expert tiles appended after the routed ones
 };
 
 cudaError_t launch_route(const RouteArgs &a, cudaStream_t s);
 cudaError_t launch_router_logits(const uint16_t *x, const float *Wg, float *h, int B, int N,
                                  int d, int32_t *done, cudaStream_t s);
 cudaError_t launch_combine(const float *out, const int32_t *pos, const float *w,
-                           const Meta *meta, uint16_t *y, int B, int d, int k,
+                           const Meta *meta, uint16_t *y, int B, int d, int k, int n_shared,
                            cudaStream_t s);
 cudaError_t launch_gather(const uint16_t *x, const int32_t *perm, const Meta *meta,
-                          uint16_t *xp, int max_pairs, int d, int k, cudaStream_t s);
+                          uint16_t *xp, int max_rows, int B, int d, int k, cudaStream_t s);
 
 struct FfnArgs {
   const uint16_t *W_gate, *W_up, *W_down;
-  const uint16_t *xp;    // [max_pairs, d] permuted token rows
-  uint16_t *act;         // [max_pairs, F] silu(g) * u, bf16
-  float *out;            // [max_pairs, d] expert outputs, fp32
+  const uint16_t *S_gate, *S_up, *S_down;   // shared experts, used when n_shared > 0
+  int n_shared;
+  const uint16_t *xp;    // [max_rows, d] permuted token rows
+  uint16_t *act;         // [max_rows, F] silu(g) * u, bf16
+  float *out;            // [max_rows, d] expert outputs, fp32
   const Tile *tiles;
   Meta *meta;
   xs_stats *stats;       // nullable
   void *part;            // partial-sum scratch
   int32_t *cnt;          // arrival counters (cleared by the routing kernel)
-  int N, d, F, max_pairs, max_tiles, n_sms;
+  int N, d, F, max_rows, max_tiles, n_sms;
 };
 
 cudaError_t launch_ffn_gate_up(const FfnArgs &a, cudaStream_t s);

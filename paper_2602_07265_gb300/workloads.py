@@ -14,7 +14,7 @@ Sec. 4 / Assumption 2; requests drawn from a few latent domains, Sec. 6.3).
 Distributions (second parameter of N(., .) is a standard deviation):
   x     : bf16, see `x_kind` below
   W_g   : fp32, N(0, 1/sqrt(d)), so a logit has variance |x|^2 / d
-  W_gate, W_up [N, F, d], W_down [N, d, F]: bf16, N(0, 0.02)
+  W_gate, W_up [N, F, d], W_down [N, d, F]: bf16, N(0, 0.02); shared experts alike
 """
 
 from __future__ import annotations
@@ -155,6 +155,13 @@ def expert_weights(w: Workload, seed: int = 0, device: str = "cuda",
             for t, shape in ((Wg, (F, d)), (Wu, (F, d)), (Wd, (d, F))):
                 t[i].copy_(torch.randn(*shape, generator=g, device=device) * EXPERT_STD)
     return Wg, Wu, Wd
+
+
+def shared_expert_weights(w: Workload, n_shared: int, seed: int = 0,
+                          device: str = "cuda") -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    """Shared experts [n_shared, F, d], [n_shared, F, d], [n_shared, d, F], bf16,
+    N(0, 0.02), from a seed stream apart from the routed experts'."""
+    return expert_weights(w.with_(N=n_shared), seed + 7_777_777, device=device)
 
 
 def random_scores(B: int, N: int, seed: int, ties: bool = False) -> np.ndarray:

@@ -38,6 +38,15 @@ class RouteParams(ctypes.Structure):
                 ("m_g", ctypes.c_int32)]
 
 
+class SharedExperts(ctypes.Structure):
+    """xs_shared_experts (device pointers and count)."""
+    _fields_ = [("W_gate", ctypes.c_void_p), ("W_up", ctypes.c_void_p),
+                ("W_down", ctypes.c_void_p), ("n_shared", ctypes.c_int32)]
+
+
+MAX_SHARED = 8
+
+
 def route_params(k0: int = 0, m_r: int = 0, tokens_per_request: int = 1, n_groups: int = 1,
                  m_g: int = 0) -> RouteParams:
     return RouteParams(k0, m_r, tokens_per_request, n_groups, m_g)
@@ -51,11 +60,12 @@ def _load() -> ctypes.CDLL:
     lib = ctypes.CDLL(path)
     P, I, Z = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
     PR = ctypes.POINTER(RouteParams)
-    lib.xshare_workspace_size.argtypes = [I, I, I, I, I, I, PR]
+    PS = ctypes.POINTER(SharedExperts)
+    lib.xshare_workspace_size.argtypes = [I, I, I, I, I, I, PR, I]
     lib.xshare_workspace_size.restype = Z
     lib.xshare_route.argtypes = [P, I, I, I, I, I, PR, P, P, P, P, P, P, P, P, Z, P]
     lib.xshare_route.restype = I
-    lib.xshare_moe_forward.argtypes = [P, P, P, P, P, I, I, I, I, I, I, I, PR,
+    lib.xshare_moe_forward.argtypes = [P, P, P, P, P, I, I, I, I, I, I, I, PR, PS,
                                        P, P, P, P, P, P, P, Z, P]
     lib.xshare_moe_forward.restype = I
     lib.xshare_route_static.argtypes = [P, I, I, I, I, I, PR, P, P, P, P, P, P, P, P]
@@ -107,9 +117,9 @@ def _check(rc: int, where: str):
 
 
 def xshare_workspace_size(B: int, N: int, k: int, d: int, F: int, mode: int,
-                          params: RouteParams) -> int:
+                          params: RouteParams, n_shared: int = 0) -> int:
     """Bytes of workspace for these sizes (d = F = 0 for xshare_route); 0 if invalid."""
-    return int(LIB.xshare_workspace_size(B, N, k, d, F, mode, ctypes.byref(params)))
+    return int(LIB.xshare_workspace_size(B, N, k, d, F, mode, ctypes.byref(params), n_shared))
 
 
 def xshare_route(scores: torch.Tensor, k: int, budget: int, mode: int, params: RouteParams,
@@ -161,11 +171,14 @@ def xshare_moe_forward(x: torch.Tensor, W_g: torch.Tensor, W_gate: torch.Tensor,
                        topk_ids: Optional[torch.Tensor] = None,
                        topk_w: Optional[torch.Tensor] = None,
                        stats: Optional[torch.Tensor] = None, stream=None,
-                       stage_events: Optional[list] = None) -> None:
-    """One MoE-layer forward (routed part) into y [B, d] bf16; see xshare.h.
+                       stage_events: Optional[list] = None,
+                       shared: Optional[tuple] = None) -> None:
+    """One MoE-layer forward into y [B, d] bf16; see xshare.h.
 
-    With `stage_events` (XS_N_STAGES + 1 torch.cuda.Event objects) the
-    profiled entry point records them between the kernel launches."""
+    `shared` = (S_gate [Ns, F, d], S_up [Ns, F, d], S_down [Ns, d, F]) bf16
+    adds the shared experts.  With `stage_events` (XS_N_STAGES + 1
+    torch.cuda.Event objects) the profiled entry point records them between
+    the kernel launches."""
     B, d = x.shape
     N = W_g.shape[0]
     F = W_gate.shape[1]
@@ -173,11 +186,22 @@ def xshare_moe_forward(x: torch.Tensor, W_g: torch.Tensor, W_gate: torch.Tensor,
             or tuple(W_down.shape) != (N, d, F) or tuple(y.shape) != (B, d):
         raise ValueError("inconsistent shapes: x [B,d], W_g [N,d], W_gate/W_up [N,F,d], "
                          "W_down [N,d,F], y [B,d]")
+    sh = None
+    if shared is not None:
+        S_gate, S_up, S_down = shared
+        Ns = S_gate.shape[0]
+        if tuple(S_gate.shape) != (Ns, F, d) or tuple(S_up.shape) != (Ns, F, d) \
+                or tuple(S_down.shape) != (Ns, d, F):
+            raise ValueError("inconsistent shared-expert shapes: [Ns,F,d], [Ns,F,d], [Ns,d,F]")
+        sh = SharedExperts(_ptr(S_gate, torch.bfloat16, "S_gate"),
+                           _ptr(S_up, torch.bfloat16, "S_up"),
+                           _ptr(S_down, torch.bfloat16, "S_down"), Ns)
     args = [
         _ptr(x, torch.bfloat16, "x"), _ptr(W_g, torch.float32, "W_g"),
         _ptr(W_gate, torch.bfloat16, "W_gate"), _ptr(W_up, torch.bfloat16, "W_up"),
         _ptr(W_down, torch.bfloat16, "W_down"), B, d, F, N, k, budget, mode,
-        ctypes.byref(params), _ptr(y, torch.bfloat16, "y"),
+        ctypes.byref(params), ctypes.byref(sh) if sh is not None else None,
+        _ptr(y, torch.bfloat16, "y"),
         _ptr(scores_out, torch.float32, "scores_out", B * N),
         _ptr(sel_mask, torch.uint8, "sel_mask", N), _ptr(topk_ids, torch.int32, "topk_ids", B * k),
         _ptr(topk_w, torch.float32, "topk_w", B * k), _ptr(stats, torch.int32, "stats", STATS_WORDS),

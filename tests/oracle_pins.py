@@ -377,6 +377,36 @@ def check_layer_single_token(O):
     assert np.allclose(r["y"][0], y.numpy(), rtol=1e-5, atol=1e-7 * float(y.abs().max()))
 
 
+def check_shared_experts(O):
+    """With shared experts, y = sum_i g_i E_i(x) + sum_j E^s_j(x) (Sec. 2.1):
+    the layer output minus the routed-only output equals the shared experts'
+    SwiGLU outputs computed with torch, for every token."""
+    g = torch.Generator().manual_seed(14)
+    N, k, d, F, B, Ns = 10, 2, 24, 16, 5, 2
+    x = bf16_round(torch.randn(B, d, generator=g))
+    W_g = torch.randn(N, d, generator=g) / math.sqrt(d)
+    Wg = bf16_round(torch.randn(N, F, d, generator=g) * 0.2)
+    Wu = bf16_round(torch.randn(N, F, d, generator=g) * 0.2)
+    Wd = bf16_round(torch.randn(N, d, F, generator=g) * 0.2)
+    Sg = bf16_round(torch.randn(Ns, F, d, generator=g) * 0.2)
+    Su = bf16_round(torch.randn(Ns, F, d, generator=g) * 0.2)
+    Sd = bf16_round(torch.randn(Ns, d, F, generator=g) * 0.2)
+    get = lambda e: (bits(Wg[e]), bits(Wu[e]), bits(Wd[e]))
+    gets = lambda j: (bits(Sg[j]), bits(Su[j]), bits(Sd[j]))
+    routed = O.moe_forward(bits(x), W_g.numpy(), get, k, 3, O.MODE_BATCH)["y"]
+    full = O.moe_forward(bits(x), W_g.numpy(), get, k, 3, O.MODE_BATCH, get_shared=gets,
+                         n_shared=Ns)["y"]
+    X = x.to(torch.float64)
+    ref = torch.zeros(B, d, dtype=torch.float64)
+    for j in range(Ns):
+        ref += (torch.nn.functional.silu(X @ Sg[j].to(torch.float64).T) *
+                (X @ Su[j].to(torch.float64).T)) @ Sd[j].to(torch.float64).T
+    assert np.allclose(full - routed, ref.numpy(), rtol=1e-10, atol=1e-12)
+    sub = O.moe_forward(bits(x), W_g.numpy(), get, k, 3, O.MODE_BATCH, tokens=[4, 0],
+                        get_shared=gets, n_shared=Ns)["y"]
+    assert np.allclose(sub, full[[4, 0]], rtol=1e-12, atol=1e-14)
+
+
 def check_combine_multi_token(O):
     """y for several tokens equals per-token sums of w * E_e(x) (Sec. 2.1) computed
     with torch, for a routing with padding slots."""
@@ -439,6 +469,6 @@ ALL_CHECKS = [
     check_closed_form_golden, check_union_statistics, check_greedy_bruteforce,
     check_hier_bruteforce, check_hier_single_request_is_batch, check_group,
     check_refine_invariants, check_zero_scores, check_budget_n_is_topk, check_permutation,
-    check_router_softmax, check_expert_ffn, check_layer_single_token,
+    check_router_softmax, check_expert_ffn, check_layer_single_token, check_shared_experts,
     check_combine_multi_token, check_canonical_sum_golden, check_canonical_sum_bound,
 ]

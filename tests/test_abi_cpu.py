@@ -89,17 +89,24 @@ def test_route_rejects_bad_params(X, prm, mode, code):
 def test_forward_rejects_bad_shapes(X):
     prm = X.route_params()
     P = 1 << 20
-    def rc(d, F, x=P, y=P):
+    def rc(d, F, x=P, y=P, shared=None):
+        sh = ctypes.byref(shared) if shared is not None else None
         return X.LIB.xshare_moe_forward(x, P, P, P, P, 4, d, F, 16, 2, 2, 1, ctypes.byref(prm),
-                                        y, None, None, None, None, None, P, 1 << 20, None)
+                                        sh, y, None, None, None, None, None, P, 1 << 20, None)
     assert rc(100, 256) == -1
     assert rc(256, 64) == -1
     assert rc(0, 256) == -1
     assert rc(256, 256, x=None) == -3
     assert rc(256, 256, y=P + 8) == -5
+    assert rc(256, 256, shared=X.SharedExperts(P, P, P, 9)) == -2
+    assert rc(256, 256, shared=X.SharedExperts(P, P, P, -1)) == -2
+    assert rc(256, 256, shared=X.SharedExperts(P, None, P, 1)) == -3
+    assert rc(256, 256, shared=X.SharedExperts(P, P, P + 2, 1)) == -5
 
 
 def test_workspace_size_rejects_invalid(X):
     prm = X.route_params()
     assert X.xshare_workspace_size(0, 16, 4, 0, 0, 1, prm) == 0
     assert X.xshare_workspace_size(8, 16, 4, 100, 256, 1, prm) == 0
+    assert X.xshare_workspace_size(8, 16, 4, 256, 256, 1, prm, 9) == 0
+    assert X.xshare_workspace_size(8, 16, 4, 0, 0, 1, prm, 1) == 0  # routing alone has none

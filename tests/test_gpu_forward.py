@@ -55,11 +55,12 @@ def device_weights(w: W.Workload, seed: int):
     return _weights_cache[key]
 
 
-def gpu_forward(X, w: W.Workload, x, W_g, weights):
+def gpu_forward(X, w: W.Workload, x, W_g, weights, shared=None):
     dev = torch.device("cuda")
     Wg, Wu, Wd = weights
     prm = X.route_params(**w.params())
-    ws = torch.empty(X.xshare_workspace_size(w.B, w.N, w.k, w.d, w.F, w.mode, prm),
+    n_shared = 0 if shared is None else shared[0].shape[0]
+    ws = torch.empty(X.xshare_workspace_size(w.B, w.N, w.k, w.d, w.F, w.mode, prm, n_shared),
                      dtype=torch.uint8, device=dev)
     out = dict(
         y=torch.empty(w.B, w.d, dtype=torch.bfloat16, device=dev),
@@ -71,7 +72,8 @@ def gpu_forward(X, w: W.Workload, x, W_g, weights):
     )
     X.xshare_moe_forward(x.to(dev), W_g.to(dev), Wg, Wu, Wd, w.k, w.budget, w.mode, prm,
                          out["y"], ws, scores_out=out["p"], sel_mask=out["mask"],
-                         topk_ids=out["ids"], topk_w=out["w"], stats=out["stats"])
+                         topk_ids=out["ids"], topk_w=out["w"], stats=out["stats"],
+                         shared=shared)
     torch.cuda.synchronize()
     r = {name: t.cpu() for name, t in out.items()}
     r["stats"] = X.stats_dict(out["stats"])
@@ -98,7 +100,7 @@ def robust_selection(p, w: W.Workload, rtol: float, trials: int = 6) -> bool:
     return True
 
 
-def compare(w, g, x, W_g, weights, tokens=None):
+def compare(w, g, x, W_g, weights, tokens=None, shared=None):
     """Check a GPU forward against the oracle; returns (ref, max_rel, fro, n_tokens_compared).
 
     The GPU decides its selection on its own fp32 scores, which differ from
@@ -112,7 +114,13 @@ def compare(w, g, x, W_g, weights, tokens=None):
     def get(e):
         return W.bf16_bits(Wg[e]), W.bf16_bits(Wu[e]), W.bf16_bits(Wd[e])
 
-    ref = O.moe_forward(xb, W_g.numpy(), get, w.k, w.budget, w.mode, tokens=tokens, **w.params())
+    extra = {}
+    if shared is not None:
+        Sg, Su, Sd = shared
+        extra = dict(n_shared=Sg.shape[0], get_shared=lambda j: (
+            W.bf16_bits(Sg[j]), W.bf16_bits(Su[j]), W.bf16_bits(Sd[j])))
+    ref = O.moe_forward(xb, W_g.numpy(), get, w.k, w.budget, w.mode, tokens=tokens,
+                        **extra, **w.params())
     rel = np.abs(g["p"].astype(np.float64) - ref["p"]) / ref["p"].astype(np.float64)
     assert rel.max() <= P_RTOL, f"scores: max relative error {rel.max():.3e}"
     toks = list(range(w.B)) if tokens is None else list(tokens)
@@ -216,3 +224,46 @@ def test_forward_deterministic(X):
     a = gpu_forward(X, w, x, W_g, weights)
     b = gpu_forward(X, w, x, W_g, weights)
     assert np.array_equal(a["y"], b["y"]) and np.array_equal(a["p"], b["p"])
+
+
+# ---- shared experts (Sec. 2.1: y = sum_i g_i E_i(x) + sum_j E^s_j(x)) ----
+SHARED = [
+    (W.TINY, 1), (W.TINY, 2), (W.TINY.with_(mode=W.MODE_TOPK), 1),
+    (W.OLMOE.with_(B=32, budget=24, k0=1), 1), (W.QWEN3, 1), (W.QWEN3.with_(B=200), 2),
+    (W.TINY.with_(B=1, budget=4, k0=1), 3),
+]
+
+
+@pytest.mark.parametrize("case", range(len(SHARED)))
+def test_forward_shared_experts_small(X, case):
+    w, ns = SHARED[case]
+    x, W_g = W.router_inputs(w, 4)
+    weights = device_weights(w, 4)
+    shared = W.shared_expert_weights(w, ns, 4)
+    g = gpu_forward(X, w, x, W_g, weights, shared=shared)
+    compare(w, g, x, W_g, weights, shared=shared)
+
+
+def test_forward_shared_experts_empty_selection(X):
+    """|S| = 0: no routed expert, y is the shared experts' output alone."""
+    w = W.TINY.with_(budget=0, k0=0)
+    x, W_g = W.router_inputs(w, 6)
+    weights = device_weights(w, 0)
+    shared = W.shared_expert_weights(w, 1, 6)
+    g = gpu_forward(X, w, x, W_g, weights, shared=shared)
+    assert g["stats"]["n_pairs"] == 0 and np.abs(g["y"]).max() > 0
+    compare(w, g, x, W_g, weights, shared=shared)
+
+
+def test_forward_shared_experts_full_size_sampled(X):
+    """DeepSeek-R1 layer with its one shared expert, sampled tokens."""
+    w = W.DSR1
+    x, W_g = W.router_inputs(w, 0)
+    weights = device_weights(w, 0)
+    shared = W.shared_expert_weights(w, 1, 0)
+    g = gpu_forward(X, w, x, W_g, weights, shared=shared)
+    compare(w, g, x, W_g, weights, tokens=[0, 13, 31], shared=shared)
+    # The routed part is unchanged by adding the shared expert.
+    g0 = gpu_forward(X, w, x, W_g, weights)
+    assert np.array_equal(g0["ids"], g["ids"]) and np.array_equal(g0["p"], g["p"])
+    assert not np.array_equal(g0["y"], g["y"])

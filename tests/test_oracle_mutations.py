@@ -144,6 +144,14 @@ def _router_transposed_input(x_bits, W_g):
     return (x[::-1] @ W.T)
 
 
+def _shared_dropped(x_bits, get_shared, n_shared, tokens):
+    return np.zeros((len(list(tokens)), x_bits.shape[1]))
+
+
+def _shared_first_only(x_bits, get_shared, n_shared, tokens):
+    return _orig["shared_experts_out"](x_bits, get_shared, min(n_shared, 1), tokens)
+
+
 def _closed_form_wrong(N, k, B):
     return N * (1.0 - (1.0 - k / N) ** (B - 1))
 
@@ -169,6 +177,8 @@ MUTATIONS = {
     "combine ignores weights": ("combine", _combine_unweighted),
     "router rows misindexed": ("router_logits", _router_transposed_input),
     "closed form exponent": ("expected_union_size", _closed_form_wrong),
+    "shared experts dropped": ("shared_experts_out", _shared_dropped),
+    "only the first shared expert": ("shared_experts_out", _shared_first_only),
 }
 
 _orig = {name: getattr(O, name) for name, _ in MUTATIONS.values()}
