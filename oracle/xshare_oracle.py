@@ -17,6 +17,7 @@ What it computes, in the paper's order and notation:
     - BATCH  : Algorithm 2 with Algorithm 1 in fixed-budget form
     - HIER   : Algorithm 4 calling Algorithm 3 per request, Eq. 3-4
     - GROUP  : Algorithm 6 calling Algorithm 5, Eq. 5
+    - THRESH : Algorithm 2 with Algorithm 1 in its threshold form (tau)
     - TOPK   : S = E, i.e. plain top-k routing (Sec. 2.2)
 * Refinement: each token routed to Top k(G_i, S) with renormalised weights
                                                             (Sec. 2.2, Algorithms 2/4/6)
@@ -44,8 +45,10 @@ MODE_TOPK = 0
 MODE_BATCH = 1
 MODE_GROUP = 2
 MODE_HIER = 3
+MODE_THRESH = 4
 
-MODE_NAMES = {MODE_TOPK: "topk", MODE_BATCH: "batch", MODE_GROUP: "group", MODE_HIER: "hier"}
+MODE_NAMES = {MODE_TOPK: "topk", MODE_BATCH: "batch", MODE_GROUP: "group", MODE_HIER: "hier",
+              MODE_THRESH: "thresh"}
 
 # Width of one chunk of the canonical column sum (one warp of 32 lanes).
 CHUNK = 32
@@ -185,6 +188,65 @@ def greedy_select_budget(scores: np.ndarray, m: int, S0: Set[int]) -> Set[int]:
             break
         S.add(ranked(scores, rest)[0])
     return S
+
+
+def expert_tree_sum(values: np.ndarray, members: Set[int]) -> np.float32:
+    """f(S) = sum of values[j] over j in S, in a fixed fp32 order.
+
+    The values of the members are placed at their expert index in a vector of
+    zeros whose length is a power of two >= N, and a halving tree is applied
+    (for o = len/2, ..., 1: v[l] <- v[l] + v[l + o] for l < o); the sum is
+    v[0].  Because x + 0 = x exactly, the padded length does not change the
+    result.  Every addition is one fp32 addition rounded to nearest.
+    """
+    values = np.asarray(values, dtype=np.float32)
+    L = 1
+    while L < values.shape[0]:
+        L *= 2
+    v = np.zeros(L, dtype=np.float32)
+    for j in members:
+        v[j] = values[j]
+    o = L // 2
+    while o >= 1:
+        v[:o] = v[:o] + v[o:2 * o]
+        o //= 2
+    return np.float32(v[0])
+
+
+def greedy_select_threshold(scores: np.ndarray, tau: float, S0: Set[int]) -> Set[int]:
+    """Algorithm 1 as printed, with a threshold tau on the covered score mass.
+
+    Starting from S_0, while f(S) < tau * f(E), add argmax_{e in E \\ S}
+    scores[e] (Algorithm 1's loop; its condition names P for G, read as the
+    scores G).  The loop also ends when E \\ S is empty.
+
+    Precision.  f(E) and f(S_0) are `expert_tree_sum`s; the target is the
+    fp32 product tau * f(E) rounded once.  When e is added, f(S) becomes the
+    fp32 sum f(S) + scores[e]: by Proposition 1 the gain of adding e is
+    exactly scores[e], whatever S is.
+    """
+    scores = np.asarray(scores, dtype=np.float32)
+    N = scores.shape[0]
+    S = set(S0)
+    target = np.float32(np.float32(tau) * expert_tree_sum(scores, set(range(N))))
+    f = expert_tree_sum(scores, S)
+    while f < target:
+        rest = [e for e in range(N) if e not in S]
+        if not rest:
+            break
+        e = ranked(scores, rest)[0]
+        S.add(e)
+        f = np.float32(f + scores[e])
+    return S
+
+
+def select_threshold(p: np.ndarray, tau: float, k0: int) -> Tuple[Set[int], Set[int]]:
+    """Algorithm 2 with GreedySelect in its threshold form: warm-up S_0, then
+    add experts until they cover a fraction tau of the batch's score mass."""
+    B = p.shape[0]
+    S0 = warmup_set(p, k0, range(B))
+    scores = canonical_column_sum(p, range(B))
+    return greedy_select_threshold(scores, tau, S0), S0
 
 
 def select_batch(p: np.ndarray, m: int, k0: int) -> Tuple[Set[int], Set[int]]:
@@ -336,13 +398,15 @@ def permute(ids: np.ndarray, N: int) -> Dict[str, np.ndarray]:
 # --------------------------------------------------------------------------
 
 def route(p: np.ndarray, k: int, budget: int, mode: int, k0: int = 0, m_r: int = 0,
-          tokens_per_request: int = 1, n_groups: int = 1, m_g: int = 0) -> Dict[str, object]:
+          tokens_per_request: int = 1, n_groups: int = 1, m_g: int = 0,
+          tau: float = 0.0) -> Dict[str, object]:
     """Batch-aware selection and refinement on fp32 gating scores p [B, N].
 
     mode TOPK : S = E (standard top-k routing, the paper's baseline)
     mode BATCH: Algorithm 2 with budget m = `budget`, warm-up k0
     mode HIER : Algorithm 4 with batch budget m = `budget`, per-request m_r, k0
     mode GROUP: Algorithm 6 with G = n_groups contiguous groups, per-group m_g, k0
+    mode THRESH: Algorithm 2 with Algorithm 1's threshold tau (fp32), k0; no budget
     Returns the selected mask, the routing, the permutation and the statistics
     |S|, |U|, |union of plain top-k| and max_g |S intersect E_g|.
     """
@@ -356,6 +420,8 @@ def route(p: np.ndarray, k: int, budget: int, mode: int, k0: int = 0, m_r: int =
         S, _ = select_hier(p, budget, m_r, k0, tokens_per_request)
     elif mode == MODE_GROUP:
         S, _ = select_group(p, n_groups, m_g, k0)
+    elif mode == MODE_THRESH:
+        S, _ = select_threshold(p, tau, k0)
     else:
         raise ValueError(f"unknown mode {mode}")
     ids, w = refine(p, S, k)

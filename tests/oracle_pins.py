@@ -15,7 +15,9 @@ the oracle disagrees with what the paper or the mathematics fixes:
   (numpy lexsort), softmax / router / SwiGLU against torch float64, the
   permutation against Python's sorted;
 * the canonical column-sum order on a hand-derived fixture, and its error
-  against the exact sum.
+  against the exact sum;
+* Algorithm 1's threshold form on a hand-derived fixture, and by brute force:
+  the smallest superset of S_0 covering a fraction tau of the score mass.
 
 `test_oracle_pins.py` runs them on the oracle; `test_oracle_mutations.py`
 plants mistakes in the oracle and checks that some pin fails.
@@ -465,10 +467,86 @@ def check_canonical_sum_bound(O, cases=20):
             assert abs(Fraction(float(got[j])) - ex[j]) <= Fraction(bound), (B, j)
 
 
+# ---------------------------------------------------------------- Algorithm 1, threshold form
+
+def check_threshold_golden(O):
+    """Hand-derived threshold selections and expert-order sums (fixture)."""
+    with open(os.path.join(GOLDEN, "threshold_example.json")) as f:
+        g = json.load(f)
+    p = np.array(g["p"], dtype=np.float32)
+    for c in g["cases"]:
+        r = O.route(p, 2, 0, O.MODE_THRESH, k0=c["k0"], tau=c["tau"])
+        assert sorted(mask_to_set(r["mask"])) == c["S"], (c, sorted(mask_to_set(r["mask"])))
+    t = g["tree_sum"]
+    v = np.array([int(h, 16) for h in t["values_hex"]], dtype=np.uint32).view(np.float32)
+    got = np.float32(O.expert_tree_sum(v, set(range(v.shape[0])))).view(np.uint32)
+    assert got == int(t["expected_hex"], 16), hex(int(got))
+    got = np.float32(O.expert_tree_sum(v, set(t["subset"]["members"]))).view(np.uint32)
+    assert got == int(t["subset"]["expected_hex"], 16), hex(int(got))
+
+
+def check_threshold_bruteforce(O, cases=40):
+    """With exact sums, the threshold selection is S_0 alone if f(S_0) already
+    reaches tau f(E); otherwise a superset of S_0 reaching tau f(E) (or all of
+    E) such that no superset of S_0 with one expert fewer reaches it, and with
+    the largest f among the supersets of its size (Corollary 1)."""
+    rng = np.random.default_rng(21)
+    done = 0
+    while done < cases:
+        N = int(rng.integers(3, 10))
+        B = int(rng.integers(1, 6))
+        k0 = int(rng.integers(0, 3))
+        tau = float(rng.integers(0, 33)) / 32.0
+        p = quantised_scores(rng, B, N)
+        col = exact_colsum(p, range(B))
+        total = sum(col, Fraction(0))
+        target = Fraction(tau) * total
+        if Fraction(float(np.float32(np.float32(tau) * np.float32(float(total))))) != target:
+            continue   # keep to cases whose target is exact in fp32
+        S0 = set()
+        for i in range(B):
+            S0 |= set(lexsort_top(p[i], k0, range(N)))
+        S = mask_to_set(O.route(p, 1, 0, O.MODE_THRESH, k0=k0, tau=tau)["mask"])
+        f = lambda A: sum((col[j] for j in A), Fraction(0))
+        assert S0 <= S
+        rest = [j for j in range(N) if j not in S0]
+        if f(S0) >= target:
+            assert S == S0
+        else:
+            assert f(S) >= target or len(S) == N
+            fewer = len(S) - len(S0) - 1
+            for c in itertools.combinations(rest, fewer):
+                assert f(S0 | set(c)) < target, (S0, c, target)
+            best = max(f(S0 | set(c)) for c in itertools.combinations(rest, len(S) - len(S0)))
+            assert f(S) == best
+        done += 1
+
+
+def check_threshold_consistency(O):
+    """On softmax scores: the threshold selection equals the fixed-budget one
+    with m = |S| - |S_0| (one greedy order), and grows with tau."""
+    rng = np.random.default_rng(5)
+    for trial in range(6):
+        B, N = int(rng.integers(1, 40)), int(rng.integers(8, 80))
+        h = rng.standard_normal((B, N)) * 1.5
+        p = (np.exp(h) / np.exp(h).sum(axis=1, keepdims=True)).astype(np.float32)
+        k0 = trial % 3
+        prev = None
+        for tau in (0.0, 0.2, 0.45, 0.7, 0.9, 1.0):
+            S = mask_to_set(O.route(p, 2, 0, O.MODE_THRESH, k0=k0, tau=tau)["mask"])
+            S0 = O.warmup_set(p, k0, range(B))
+            Sb = mask_to_set(O.route(p, 2, len(S) - len(S0), O.MODE_BATCH, k0=k0)["mask"])
+            assert S == Sb, (tau, len(S), len(Sb))
+            if prev is not None:
+                assert prev <= S
+            prev = S
+
+
 ALL_CHECKS = [
     check_closed_form_golden, check_union_statistics, check_greedy_bruteforce,
     check_hier_bruteforce, check_hier_single_request_is_batch, check_group,
     check_refine_invariants, check_zero_scores, check_budget_n_is_topk, check_permutation,
     check_router_softmax, check_expert_ffn, check_layer_single_token, check_shared_experts,
     check_combine_multi_token, check_canonical_sum_golden, check_canonical_sum_bound,
+    check_threshold_golden, check_threshold_bruteforce, check_threshold_consistency,
 ]

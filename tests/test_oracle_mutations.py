@@ -152,6 +152,39 @@ def _shared_first_only(x_bits, get_shared, n_shared, tokens):
     return _orig["shared_experts_out"](x_bits, get_shared, min(n_shared, 1), tokens)
 
 
+def _threshold_non_strict(scores, tau, S0):
+    scores = np.asarray(scores, dtype=np.float32)
+    N = scores.shape[0]
+    S = set(S0)
+    target = np.float32(np.float32(tau) * O.expert_tree_sum(scores, set(range(N))))
+    f = O.expert_tree_sum(scores, S)
+    while f <= target and len(S) < N:
+        e = O.ranked(scores, [j for j in range(N) if j not in S])[0]
+        S.add(e)
+        f = np.float32(f + scores[e])
+    return S
+
+
+def _threshold_ignores_s0_mass(scores, tau, S0):
+    scores = np.asarray(scores, dtype=np.float32)
+    N = scores.shape[0]
+    S = set(S0)
+    target = np.float32(np.float32(tau) * O.expert_tree_sum(scores, set(range(N))))
+    f = np.float32(0.0)
+    while f < target and len(S) < N:
+        e = O.ranked(scores, [j for j in range(N) if j not in S])[0]
+        S.add(e)
+        f = np.float32(f + scores[e])
+    return S
+
+
+def _tree_sum_left_to_right(values, members):
+    acc = np.float32(0.0)
+    for j in sorted(members):
+        acc = np.float32(acc + np.float32(values[j]))
+    return acc
+
+
 def _closed_form_wrong(N, k, B):
     return N * (1.0 - (1.0 - k / N) ** (B - 1))
 
@@ -179,6 +212,9 @@ MUTATIONS = {
     "closed form exponent": ("expected_union_size", _closed_form_wrong),
     "shared experts dropped": ("shared_experts_out", _shared_dropped),
     "only the first shared expert": ("shared_experts_out", _shared_first_only),
+    "threshold loop runs while f <= target": ("greedy_select_threshold", _threshold_non_strict),
+    "threshold ignores the warm-up mass": ("greedy_select_threshold", _threshold_ignores_s0_mass),
+    "expert sum left to right": ("expert_tree_sum", _tree_sum_left_to_right),
 }
 
 _orig = {name: getattr(O, name) for name, _ in MUTATIONS.values()}
