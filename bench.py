@@ -63,6 +63,7 @@ def parse_args(argv=None):
     ap.add_argument("--budget", type=int, default=None)
     ap.add_argument("--k0", type=int, default=None)
     ap.add_argument("--mode", default=None, choices=sorted(W.MODES))
+    ap.add_argument("--tau", type=float, default=None, help="covered score-mass fraction (thresh)")
     ap.add_argument("--shared", type=int, default=0,
                     help="shared experts added to every token (DeepSeek-R1 has one)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -85,11 +86,14 @@ def workload_from_args(args) -> W.Workload:
         kw["k0"] = args.k0
     if args.mode is not None:
         kw["mode"] = W.MODES[args.mode]
+    if args.tau is not None:
+        kw["tau"] = args.tau
     return w.with_(**kw) if kw else w
 
 
 def describe(w: W.Workload, n_shared: int = 0) -> str:
-    mode = {0: "TOPK", 1: "BATCH (Algorithm 2)", 2: "GROUP (Algorithm 6)", 3: "HIER (Algorithm 4)"}[w.mode]
+    mode = {0: "TOPK", 1: "BATCH (Algorithm 2)", 2: "GROUP (Algorithm 6)", 3: "HIER (Algorithm 4)",
+            4: "THRESH (Algorithm 2, Algorithm 1 threshold)"}[w.mode]
     s = f"{w.name}: N={w.N} k={w.k} d={w.d} F={w.F} B={w.B} {mode}"
     if w.mode == W.MODE_BATCH:
         s += f" m={w.budget} k0={w.k0}"
@@ -97,6 +101,8 @@ def describe(w: W.Workload, n_shared: int = 0) -> str:
         s += f" m={w.budget} m_r={w.m_r} k0={w.k0} tokens/request={w.tokens_per_request}"
     elif w.mode == W.MODE_GROUP:
         s += f" G={w.n_groups} m_g={w.m_g} k0={w.k0}"
+    elif w.mode == W.MODE_THRESH:
+        s += f" tau={w.tau} k0={w.k0}"
     if n_shared:
         s += f" + {n_shared} shared expert{'s' if n_shared > 1 else ''}"
     return s
@@ -495,7 +501,7 @@ def cpu_baseline(w: W.Workload, seed: int, n_shared: int = 0) -> dict:
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
                CUDA_VISIBLE_DEVICES="")
     f_rows = max(128, w.F // 4)
-    kw = json.dumps(dict(B=w.B, budget=w.budget, k0=w.k0, mode=w.mode))
+    kw = json.dumps(dict(B=w.B, N=w.N, F=w.F, budget=w.budget, k0=w.k0, mode=w.mode, tau=w.tau))
     code = (f"import sys, json; sys.path.insert(0, {ROOT!r}); import torch; torch.set_num_threads(1); "
             f"import bench; from paper_2602_07265_gb300 import workloads as W; "
             f"w = W.WORKLOADS[{w.name!r}].with_(**{kw}); "

@@ -55,6 +55,15 @@ typedef struct CUstream_st *xs_stream_t;
  *                  S_r = S0_r + Top m_r of the request's column scores; then
  *                  S = union S_r plus the `budget` best remaining experts by the
  *                  batch column score (Sec. 4, Eq. 3-4).
+ *   XS_MODE_THRESH: Algorithm 2 with GreedySelect in the threshold form that
+ *                  Algorithm 1 prints: warm-up S_0, then while
+ *                  f(S) < tau * f(E) add the best expert of E \ S by column
+ *                  score, f(S) = sum over S of the column scores (Eq. 2).
+ *                  `budget` is ignored.  f(E) and f(S_0) are fp32 halving
+ *                  trees over the expert index (values at their index in a
+ *                  zero vector of power-of-two length, v[l] += v[l+o] for
+ *                  o = len/2 .. 1); the target is the fp32 product tau * f(E);
+ *                  adding e adds scores[e] to f(S) in fp32 (Proposition 1).
  * Ordering everywhere: larger score first, equal scores -> lower expert index.
  * Column scores are fp32 sums in a fixed order: rows in chunks of 32 (last one
  * zero-padded), a halving tree v[l] += v[l+o], o = 16, 8, 4, 2, 1, inside a
@@ -63,7 +72,8 @@ enum {
   XS_MODE_TOPK = 0,
   XS_MODE_BATCH = 1,
   XS_MODE_GROUP = 2,
-  XS_MODE_HIER = 3
+  XS_MODE_HIER = 3,
+  XS_MODE_THRESH = 4
 };
 
 /* Selection parameters (fields a mode does not use are ignored). */
@@ -74,6 +84,7 @@ typedef struct {
   int32_t n_groups;           /* GROUP: G (Sec. 5); N % G == 0.  Also used by the
                                  max_group_load statistic in every mode; 0 = 1 */
   int32_t m_g;                /* GROUP: per-group budget m_g (Algorithm 5) */
+  float tau;                  /* THRESH: covered fraction of the score mass, 0 <= tau <= 1 */
 } xs_route_params;
 
 /* Per-call statistics, written by the device into caller memory. */
@@ -90,7 +101,7 @@ typedef struct {
 /* Host-side error codes (return values). */
 #define XS_OK 0
 #define XS_ERR_SHAPE (-1)     /* B, N, k, d or F out of range or misaligned */
-#define XS_ERR_PARAM (-2)     /* mode, budget, k0, m_r, m_g, n_groups or tokens_per_request invalid */
+#define XS_ERR_PARAM (-2)     /* mode, budget, k0, m_r, m_g, n_groups, tokens_per_request or tau invalid */
 #define XS_ERR_NULL (-3)      /* a required pointer is NULL */
 #define XS_ERR_WORKSPACE (-4) /* workspace NULL, too small or not 256-byte aligned */
 #define XS_ERR_ALIGN (-5)     /* a tensor pointer is not 16-byte aligned */
@@ -123,7 +134,7 @@ size_t xshare_workspace_size(int B, int N, int k, int d, int F, int mode,
  *   scores   [B, N] fp32, device: gating scores g_ij (e.g. the dense softmax
  *            of the router logits, Sec. 2.2).
  *   budget   m: experts the greedy step adds beyond the warm-up set
- *            (BATCH, HIER); ignored by TOPK and GROUP.
+ *            (BATCH, HIER); ignored by TOPK, GROUP and THRESH.
  *   sel_mask [N] uint8, device, out: 1 for experts in S.
  *   topk_ids [B, k] int32, device, out: per token the min(k, |S|) best experts
  *            of S, best first (Top k(G_i, S), Algorithms 2, 4, 6); unused slots -1.

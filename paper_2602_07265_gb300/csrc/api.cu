@@ -42,7 +42,8 @@ int current_device_sms() {
 int check_route_args(int B, int N, int k, int budget, int mode, const xs_route_params *prm) {
   if (prm == nullptr) return XS_ERR_NULL;
   if (B < 1 || B > kMaxB || N < 1 || N > kMaxN || k < 1 || k > kMaxK || k > N) return XS_ERR_SHAPE;
-  if (mode < XS_MODE_TOPK || mode > XS_MODE_HIER) return XS_ERR_PARAM;
+  if (mode < XS_MODE_TOPK || mode > XS_MODE_THRESH) return XS_ERR_PARAM;
+  if (mode == XS_MODE_THRESH && !(prm->tau >= 0.f && prm->tau <= 1.f)) return XS_ERR_PARAM;
   if (budget < 0 || prm->k0 < 0 || prm->k0 > kMaxK || prm->k0 > N || prm->m_r < 0 || prm->m_g < 0 ||
       prm->n_groups < 0)
     return XS_ERR_PARAM;
@@ -81,6 +82,7 @@ RouteArgs route_args(const Plan &pl, void *ws, int B, int N, int k, int budget, 
   a.T = prm->tokens_per_request < 1 ? 1 : prm->tokens_per_request;
   a.G = prm->n_groups < 1 ? 1 : prm->n_groups;
   a.m_g = prm->m_g > N ? N : prm->m_g;
+  a.tau = prm->tau;
   a.p = at<float>(ws, pl.p);
   a.mask = at<uint8_t>(ws, pl.mask);
   a.ids = at<int32_t>(ws, pl.ids);

@@ -1,10 +1,10 @@
 // Router, batch-aware expert selection, refinement, permutation, gather and
 // combine kernels (steps a1-a7 and a9 of the MoE-layer forward).
 //
-// Selection follows XShare (arxiv 2602.07265): Algorithm 2 (BATCH),
-// Algorithms 3-4 (HIER), Algorithms 5-6 (GROUP) and plain top-k (TOPK), on
-// fp32 gating scores, with the refinement "route x_i to Top k(G_i, S)" and
-// the renormalised weights of Sec. 2.2.
+// Selection follows XShare (arxiv 2602.07265): Algorithm 2 (BATCH; THRESH
+// with Algorithm 1's threshold), Algorithms 3-4 (HIER), Algorithms 5-6
+// (GROUP) and plain top-k (TOPK), on fp32 gating scores, with the refinement
+// "route x_i to Top k(G_i, S)" and the renormalised weights of Sec. 2.2.
 #include <cuda_bf16.h>
 
 #include <climits>
@@ -116,6 +116,24 @@ __device__ __forceinline__ int lane_take(LaneList<Q> &L, int count, Emit emit) {
     }
   }
   return r;
+}
+
+// Halving tree over the expert index of values held as v[q] = value of expert
+// lane + 32 q (zero where there is none): for o = 16 Q, ..., 32 the pairs
+// (j, j + o) are in one lane; for o = 16, ..., 1 they are lanes l and l + o.
+// Returns the sum on every lane.  Zero padding adds exactly, so the result is
+// that of the tree over any power-of-two length >= the number of experts.
+template <int Q>
+__device__ __forceinline__ float expert_tree(float (&v)[Q]) {
+#pragma unroll
+  for (int h = Q / 2; h >= 1; h >>= 1) {
+#pragma unroll
+    for (int q = 0; q < h; ++q) v[q] = __fadd_rn(v[q], v[q + h]);
+  }
+  float x = v[0];
+#pragma unroll
+  for (int o = 16; o; o >>= 1) x = __fadd_rn(x, __shfl_down_sync(kFull, x, o));
+  return __shfl_sync(kFull, x, 0);
 }
 
 // Loads candidates j = j0 + lane + 32 q in [j0, j0 + n) with keys from
@@ -638,6 +656,36 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
           if (lane == 0) s_mask[id] = 1;
         });
       }
+  } else if (a.mode == XS_MODE_THRESH) {
+    // Algorithm 1 as printed: add the best remaining expert while the
+    // covered mass f(S) is below tau f(E); by Proposition 1 adding e adds
+    // scores[e] to f(S).
+    if (warp == 0) {
+      float vE[kQ], v0[kQ];
+#pragma unroll
+      for (int q = 0; q < kQ; ++q) {
+        const int j = lane + 32 * q;
+        vE[q] = (j < N) ? s_col[j] : 0.f;
+        v0[q] = (j < N && s_base[j]) ? s_col[j] : 0.f;
+      }
+      const float target = __fmul_rn(a.tau, expert_tree<kQ>(vE));
+      float f = expert_tree<kQ>(v0);
+      LaneList<kQ> L;
+      lane_load<kQ>(L, 0, N, lane, [&](int, int j) { return s_col[j]; },
+                    [&](int, int j) { return s_base[j] == 0; });
+      lane_sort<kQ>(L);
+      while (f < target) {
+        float v = 0.f;
+        int id = -1;
+        if (lane_take<kQ>(L, 1, [&](int, int e, float sv) {
+              id = e;
+              v = sv;
+            }) == 0)
+          break;
+        if (lane == 0) s_mask[id] = 1;
+        f = __fadd_rn(f, v);
+      }
+    }
   } else if (warp == 0) {
     // BATCH (Algorithm 2) and the batch step of HIER (Algorithm 4): add the
     // `budget` best experts outside the base set by the batch column score.

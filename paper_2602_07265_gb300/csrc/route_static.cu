@@ -60,7 +60,8 @@ extern "C" int xshare_route_static(const float *scores, int B, int N, int k, int
   if (prm == nullptr) return XS_ERR_NULL;
   if (B < 1 || B > kStaticMaxB || N < 1 || N > kMaxN || k < 1 || k > kMaxK || k > N)
     return XS_ERR_SHAPE;
-  if (mode < XS_MODE_TOPK || mode > XS_MODE_HIER) return XS_ERR_PARAM;
+  if (mode < XS_MODE_TOPK || mode > XS_MODE_THRESH) return XS_ERR_PARAM;
+  if (mode == XS_MODE_THRESH && !(prm->tau >= 0.f && prm->tau <= 1.f)) return XS_ERR_PARAM;
   if (budget < 0 || prm->k0 < 0 || prm->k0 > kMaxK || prm->k0 > N || prm->m_r < 0 ||
       prm->m_g < 0 || prm->n_groups < 0)
     return XS_ERR_PARAM;
@@ -101,6 +102,7 @@ extern "C" int xshare_route_static(const float *scores, int B, int N, int k, int
   a.T = prm->tokens_per_request < 1 ? 1 : prm->tokens_per_request;
   a.G = prm->n_groups < 1 ? 1 : prm->n_groups;
   a.m_g = prm->m_g > N ? N : prm->m_g;
+  a.tau = prm->tau;
   a.mask = sel_mask;
   a.ids = topk_ids;
   a.w = topk_w;

@@ -91,6 +91,7 @@ struct RouteArgs {
   const float *logits;   // nullable: if set, p = softmax(logits) is computed first
   float *p;              // [B, N] scores (input if logits == nullptr, else output)
   int B, N, k, budget, mode, k0, m_r, T, G, m_g;
+  float tau;             // THRESH: covered fraction of the score mass
   uint8_t *mask;         // [N]
   int32_t *ids;          // [B, k]
   float *w;              // [B, k]

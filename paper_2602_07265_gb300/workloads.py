@@ -25,8 +25,9 @@ from typing import Dict, Optional, Tuple
 import numpy as np
 import torch
 
-MODE_TOPK, MODE_BATCH, MODE_GROUP, MODE_HIER = 0, 1, 2, 3
-MODES = {"topk": MODE_TOPK, "batch": MODE_BATCH, "group": MODE_GROUP, "hier": MODE_HIER}
+MODE_TOPK, MODE_BATCH, MODE_GROUP, MODE_HIER, MODE_THRESH = 0, 1, 2, 3, 4
+MODES = {"topk": MODE_TOPK, "batch": MODE_BATCH, "group": MODE_GROUP, "hier": MODE_HIER,
+         "thresh": MODE_THRESH}
 
 EXPERT_STD = 0.02
 
@@ -47,6 +48,7 @@ class Workload:
     tokens_per_request: int = 1   # 1 + L_s
     n_groups: int = 1   # G (GROUP)
     m_g: int = 0        # per-group budget (GROUP)
+    tau: float = 0.0    # covered score-mass fraction (THRESH)
     x_kind: str = "iid"  # "iid" | "request" | "domains"
     n_domains: int = 4
     domain_std: float = 1.5
@@ -55,7 +57,7 @@ class Workload:
 
     def params(self) -> Dict[str, int]:
         return dict(k0=self.k0, m_r=self.m_r, tokens_per_request=self.tokens_per_request,
-                    n_groups=self.n_groups, m_g=self.m_g)
+                    n_groups=self.n_groups, m_g=self.m_g, tau=self.tau)
 
     def with_(self, **kw) -> "Workload":
         return dataclasses.replace(self, **kw)

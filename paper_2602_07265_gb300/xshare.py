@@ -35,7 +35,7 @@ class RouteParams(ctypes.Structure):
     """xs_route_params."""
     _fields_ = [("k0", ctypes.c_int32), ("m_r", ctypes.c_int32),
                 ("tokens_per_request", ctypes.c_int32), ("n_groups", ctypes.c_int32),
-                ("m_g", ctypes.c_int32)]
+                ("m_g", ctypes.c_int32), ("tau", ctypes.c_float)]
 
 
 class SharedExperts(ctypes.Structure):
@@ -48,8 +48,8 @@ MAX_SHARED = 8
 
 
 def route_params(k0: int = 0, m_r: int = 0, tokens_per_request: int = 1, n_groups: int = 1,
-                 m_g: int = 0) -> RouteParams:
-    return RouteParams(k0, m_r, tokens_per_request, n_groups, m_g)
+                 m_g: int = 0, tau: float = 0.0) -> RouteParams:
+    return RouteParams(k0, m_r, tokens_per_request, n_groups, m_g, tau)
 
 
 def _load() -> ctypes.CDLL:

@@ -67,7 +67,7 @@ def _route_rc(X, B=8, N=16, k=4, budget=4, mode=1, prm=None, scores=1 << 20, mas
 @pytest.mark.parametrize("kw,code", [
     (dict(B=0), -1), (dict(B=8193), -1), (dict(N=0), -1), (dict(N=1025), -1),
     (dict(k=0), -1), (dict(k=17), -1), (dict(N=4, k=5), -1),
-    (dict(mode=4), -2), (dict(mode=-1), -2), (dict(budget=-1), -2),
+    (dict(mode=5), -2), (dict(mode=-1), -2), (dict(budget=-1), -2),
     (dict(scores=None), -3), (dict(mask=None), -3), (dict(ids=None), -3), (dict(w=None), -3),
     (dict(scores=(1 << 20) + 4), -5),
     (dict(ws=None), -4), (dict(ws=(1 << 20) + 16), -4),
@@ -81,6 +81,8 @@ def test_route_rejects_bad_arguments(X, kw, code):
     (dict(n_groups=0), 2, -2), (dict(n_groups=3), 2, -2), (dict(n_groups=32), 2, -2),
     (dict(tokens_per_request=0), 3, -2), (dict(tokens_per_request=3), 3, -2),
     (dict(tokens_per_request=16), 3, -2),
+    (dict(tau=-0.1), 4, -2), (dict(tau=1.5), 4, -2), (dict(tau=float("nan")), 4, -2),
+    (dict(), 5, -2),
 ])
 def test_route_rejects_bad_params(X, prm, mode, code):
     assert _route_rc(X, mode=mode, prm=X.route_params(**prm)) == code

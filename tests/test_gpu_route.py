@@ -30,7 +30,8 @@ def X():
 def gpu_route(X, p: np.ndarray, k: int, budget: int, mode: int, **params):
     B, N = p.shape
     dev = torch.device("cuda")
-    prm = X.route_params(**{**dict(k0=0, m_r=0, tokens_per_request=1, n_groups=1, m_g=0), **params})
+    prm = X.route_params(**{**dict(k0=0, m_r=0, tokens_per_request=1, n_groups=1, m_g=0, tau=0.0),
+                            **params})
     ws = torch.empty(X.xshare_workspace_size(B, N, k, 0, 0, mode, prm), dtype=torch.uint8, device=dev)
     scores = torch.from_numpy(np.ascontiguousarray(p)).to(dev)
     out = dict(
@@ -74,7 +75,7 @@ def oracle_scores(w: W.Workload, seed: int) -> np.ndarray:
 
 
 def check(X, p, k, budget, mode, **params):
-    full = dict(k0=0, m_r=0, tokens_per_request=1, n_groups=1, m_g=0)
+    full = dict(k0=0, m_r=0, tokens_per_request=1, n_groups=1, m_g=0, tau=0.0)
     full.update(params)
     ref = O.route(p, k, budget, mode, **full)
     g = gpu_route(X, p, k, budget, mode, **full)
@@ -178,3 +179,51 @@ def test_repeatable(X):
     b = gpu_route(X, p, 8, 32, W.MODE_BATCH, k0=1)
     for key in ("mask", "ids", "w", "perm", "counts"):
         assert np.array_equal(a[key], b[key]), key
+
+
+# ---- Algorithm 1 in its threshold form ----
+TAUS = [0.0, 0.25, 0.5, 0.8, 0.95, 1.0]
+
+
+@pytest.mark.parametrize("tau", TAUS)
+@pytest.mark.parametrize("name", ["tiny", "olmoe", "qwen3", "dsr1", "dsr1_group"])
+def test_threshold_route_parity(X, name, tau):
+    w = W.WORKLOADS[name]
+    for k0, seed in ((0, 0), (1, 1)):
+        p = oracle_scores(w, seed)
+        check(X, p, w.k, 0, W.MODE_THRESH, k0=k0, tau=tau,
+              n_groups=w.n_groups)
+
+
+@pytest.mark.parametrize("B,N,k,k0,tau,ties", [
+    (1, 64, 8, 0, 0.5, False),
+    (32, 50, 8, 1, 0.6, False),        # N not a multiple of 32
+    (40, 1000, 16, 2, 0.7, False),     # 32 candidates per lane
+    (96, 1024, 8, 0, 0.99, True),      # tie-heavy, nearly all the mass
+    (64, 256, 8, 0, 1.0, True),        # tau = 1: every expert
+    (2048, 256, 8, 1, 0.4, False),     # many chunks
+    (8192, 64, 2, 0, 0.3, True),       # B at the limit
+    (33, 128, 4, 4, 0.0, False),       # tau = 0: the warm-up set alone
+])
+def test_threshold_edge_cases(X, B, N, k, k0, tau, ties):
+    p = W.random_scores(B, N, seed=B + N + k0, ties=ties)
+    check(X, p, k, 0, W.MODE_THRESH, k0=k0, tau=tau)
+
+
+def test_threshold_tau_grid_bit_exact(X):
+    """Many tau values on one score matrix: every |S| from the warm-up set to
+    N is met, so each stopping point is compared."""
+    p = W.random_scores(48, 128, seed=11)
+    sizes = set()
+    for i in range(41):
+        ref = check(X, p, 8, 0, W.MODE_THRESH, k0=1, tau=i / 40.0)
+        sizes.add(ref["n_selected"])
+    assert len(sizes) > 20
+
+
+def test_threshold_zero_scores(X):
+    p = W.random_scores(16, 64, seed=2)
+    p[:, 10:] = 0.0
+    check(X, p, 8, 0, W.MODE_THRESH, k0=0, tau=1.0)
+    p[:] = 0.0
+    check(X, p, 8, 0, W.MODE_THRESH, k0=0, tau=0.5)

@@ -48,6 +48,8 @@ def test_route_static_matches_route_twice(X):
          X.route_params(k0=1, m_r=4, tokens_per_request=4)),
         (W.random_scores(32, 64, seed=42, ties=True), 8, 12, W.MODE_BATCH,
          X.route_params(k0=1)),
+        (W.random_scores(96, 128, seed=43), 8, 0, W.MODE_THRESH,
+         X.route_params(k0=1, tau=0.6)),
     ]
     for p, k, budget, mode, prm in cases:
         B, N = p.shape
