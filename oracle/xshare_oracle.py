@@ -23,7 +23,9 @@ What it computes, in the paper's order and notation:
                                                             (Sec. 2.2, Algorithms 2/4/6)
 * Permutation of (token, slot) pairs by expert (counting sort, stable)
 * Expert FFN E_i(x) = W_down (silu(W_gate x) * (W_up x)) over the pairs, and the
-  weighted combine y = sum_i g_i(x) E_i(x) of the routed part  (Sec. 2.1)
+  weighted combine y = sum_i g_i(x) E_i(x) + sum_j E^s_j(x)   (Sec. 2.1)
+* A stack of L residual MoE layers with the global budget split m_l = K / L
+                                                            (Eq. 1, Sec. 3.2)
 
 Precision.  Selection is decided on fp32 scores (the precision the kernels
 decide in): softmax is evaluated in fp64 and rounded to fp32 once, column sums
@@ -66,6 +68,21 @@ def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
     """
     b = np.asarray(bits, dtype=np.uint16)
     return (b.astype(np.uint32) << np.uint32(16)).view(np.float32).astype(np.float64)
+
+
+def f64_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round float64 values to bf16 (8 significant bits, fp32's exponent range),
+    to nearest with ties to even, in one step.  Returns uint16 bit patterns.
+
+    x = m 2^e with 0.5 <= |m| < 1; the bf16 quantum at that binade is
+    2^(e - 8), or 2^-133 below the normal range (e < -125).  np.rint rounds
+    half to even.  Values beyond bf16's range are not expected here.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    _, e = np.frexp(x)
+    q = np.maximum(e, -125) - 8
+    r = np.ldexp(np.rint(np.ldexp(x, -q)), q)
+    return (r.astype(np.float32).view(np.uint32) >> np.uint32(16)).astype(np.uint16)
 
 
 # --------------------------------------------------------------------------
@@ -543,6 +560,45 @@ def moe_forward(x_bits: np.ndarray, W_g: np.ndarray, get_expert, k: int, budget:
         y = y + shared_experts_out(x_bits, get_shared, n_shared, toks)
     r["y"] = y
     return r
+
+
+# --------------------------------------------------------------------------
+# Eq. 1 at the system level: a stack of L MoE layers under a global budget
+# --------------------------------------------------------------------------
+
+def layer_budgets(K: int, L: int) -> List[int]:
+    """Uniform split m_l = K / L of the global budget K (Sec. 3.2, Eq. 1).
+
+    Reading: K is split into integers that sum to K, the first K mod L
+    layers taking one more: m_l = floor(K / L) + (1 if l < K mod L else 0).
+    """
+    return [K // L + (1 if l < K % L else 0) for l in range(L)]
+
+
+def moe_stack_forward(x_bits: np.ndarray, layers: Sequence[dict], k: int, K: int, mode: int,
+                      stats: Optional[list] = None, **params) -> List[np.ndarray]:
+    """L residual MoE layers, x_{l+1} = x_l + MoE_l(x_l), each with budget m_l.
+
+    layers[l] = {"W_g": [N, d] fp32, "get_expert": e -> bf16 patterns,
+    optional "get_shared", "n_shared"}.  Each layer runs `moe_forward` on
+    all tokens with budget layer_budgets(K, L)[l] (the modes that take no
+    budget ignore it); the sum x_l + MoE_l(x_l) is formed in fp64 and rounded
+    once to bf16, the precision activations have between layers.  Returns the
+    bf16 patterns of x_1 .. x_L; with `stats` (a list) each layer's routing
+    dictionary is appended to it.
+    """
+    budgets = layer_budgets(K, len(layers))
+    outs = []
+    x = np.asarray(x_bits, dtype=np.uint16)
+    for l, layer in enumerate(layers):
+        r = moe_forward(x, layer["W_g"], layer["get_expert"], k, budgets[l], mode,
+                        get_shared=layer.get("get_shared"), n_shared=layer.get("n_shared", 0),
+                        **params)
+        x = f64_to_bf16_bits(bf16_bits_to_f64(x) + r["y"])
+        outs.append(x)
+        if stats is not None:
+            stats.append(r)
+    return outs
 
 
 def expected_union_size(N: int, k: int, B: int) -> float:

@@ -17,7 +17,10 @@ the oracle disagrees with what the paper or the mathematics fixes:
 * the canonical column-sum order on a hand-derived fixture, and its error
   against the exact sum;
 * Algorithm 1's threshold form on a hand-derived fixture, and by brute force:
-  the smallest superset of S_0 covering a fraction tau of the score mass.
+  the smallest superset of S_0 covering a fraction tau of the score mass;
+* the layer stack of Eq. 1: the budget split, bf16 rounding against torch and
+  hand-derived double-rounding cases, the residual identity, budget = N per
+  layer as a plain top-k stack.
 
 `test_oracle_pins.py` runs them on the oracle; `test_oracle_mutations.py`
 plants mistakes in the oracle and checks that some pin fails.
@@ -542,6 +545,71 @@ def check_threshold_consistency(O):
             prev = S
 
 
+# ---------------------------------------------------------------- Eq. 1: layer stack
+
+def check_bf16_rounding(O):
+    """Round-to-nearest-even to bf16: equals torch's fp32 -> bf16 on fp32 values
+    (ties and subnormals included), and rounds fp64 values once (hand-derived
+    cases where rounding through fp32 first would differ)."""
+    rng = np.random.default_rng(3)
+    v = (rng.standard_normal(20000) * np.exp(rng.uniform(-40, 40, 20000))).astype(np.float32)
+    base = torch.from_numpy(v).to(torch.bfloat16).to(torch.float32).numpy()
+    ties = (base.astype(np.float64) * (1 + 2.0 ** -8)).astype(np.float32)   # halfway points
+    sub = (rng.standard_normal(2000) * 2.0 ** -130).astype(np.float32)
+    for vals in (v, ties, sub):
+        want = torch.from_numpy(vals).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+        got = O.f64_to_bf16_bits(vals.astype(np.float64))
+        assert np.array_equal(got, want)
+    # 1 + 2^-8 + 2^-30: above the tie between 1 and 1 + 2^-7 -> 1 + 2^-7 (0x3f81);
+    # through fp32 first it becomes the tie 1 + 2^-8 and then 1.0 (even).
+    # -(1 + 3 * 2^-8 - 2^-40): below the tie between 1 + 2^-7 and 1 + 2^-6 -> 0xbf81.
+    got = O.f64_to_bf16_bits(np.array([1 + 2.0 ** -8 + 2.0 ** -30, -(1 + 3 * 2.0 ** -8 - 2.0 ** -40)]))
+    assert list(got) == [0x3F81, 0xBF81], [hex(int(g)) for g in got]
+
+
+def check_layer_budgets(O):
+    """m_l = K / L (Sec. 3.2): integers summing to K that differ by at most one,
+    larger first."""
+    assert O.layer_budgets(10, 4) == [3, 3, 2, 2]
+    assert O.layer_budgets(24 * 58, 58) == [24] * 58
+    assert O.layer_budgets(3, 5) == [1, 1, 1, 0, 0]
+    for K in range(0, 60):
+        for L in range(1, 9):
+            m = O.layer_budgets(K, L)
+            assert sum(m) == K and max(m) - min(m) <= 1 and m == sorted(m, reverse=True)
+
+
+def _tiny_stack(seed, L, N, d, F, zero=False):
+    g = torch.Generator().manual_seed(seed)
+    layers = []
+    for _ in range(L):
+        Wg = bf16_round(torch.randn(N, F, d, generator=g) * 0.2)
+        Wu = bf16_round(torch.randn(N, F, d, generator=g) * 0.2)
+        Wd = bf16_round(torch.randn(N, d, F, generator=g) * (0.0 if zero else 0.2))
+        W_g = (torch.randn(N, d, generator=g) / math.sqrt(d)).numpy()
+        layers.append({"W_g": W_g, "get_expert": (lambda e, Wg=Wg, Wu=Wu, Wd=Wd:
+                                                  (bits(Wg[e]), bits(Wu[e]), bits(Wd[e])))})
+    return layers
+
+
+def check_stack_invariants(O):
+    """Residual identity with zero expert outputs; each layer gets budget m_l
+    (|S_l| = m_l with k0 = 0); budget N in every layer is a plain top-k stack."""
+    B, N, d, F, k, L = 6, 8, 16, 8, 2, 3
+    x = bits(bf16_round(torch.randn(B, d, generator=torch.Generator().manual_seed(1))))
+    zero = _tiny_stack(2, L, N, d, F, zero=True)
+    outs = O.moe_stack_forward(x, zero, k, 7, O.MODE_BATCH)
+    assert all(np.array_equal(o, x) for o in outs)
+    layers = _tiny_stack(3, L, N, d, F)
+    st = []
+    O.moe_stack_forward(x, layers, k, 7, O.MODE_BATCH, stats=st)
+    assert [r["n_selected"] for r in st] == O.layer_budgets(7, L) == [3, 2, 2]
+    a = O.moe_stack_forward(x, layers, k, N * L, O.MODE_BATCH)
+    b = O.moe_stack_forward(x, layers, k, 0, O.MODE_TOPK)
+    assert all(np.array_equal(p, q) for p, q in zip(a, b))
+    assert not np.array_equal(a[-1], x)
+
+
 ALL_CHECKS = [
     check_closed_form_golden, check_union_statistics, check_greedy_bruteforce,
     check_hier_bruteforce, check_hier_single_request_is_batch, check_group,
@@ -549,4 +617,5 @@ ALL_CHECKS = [
     check_router_softmax, check_expert_ffn, check_layer_single_token, check_shared_experts,
     check_combine_multi_token, check_canonical_sum_golden, check_canonical_sum_bound,
     check_threshold_golden, check_threshold_bruteforce, check_threshold_consistency,
+    check_bf16_rounding, check_layer_budgets, check_stack_invariants,
 ]

@@ -185,6 +185,20 @@ def _tree_sum_left_to_right(values, members):
     return acc
 
 
+def _budgets_floor(K, L):
+    return [K // L] * L
+
+
+def _bf16_truncate(x):
+    x = np.asarray(x, dtype=np.float64)
+    return (x.astype(np.float32).view(np.uint32) >> np.uint32(16)).astype(np.uint16)
+
+
+def _bf16_via_fp32(x):
+    x = np.asarray(x, dtype=np.float64).astype(np.float32)
+    return _orig["f64_to_bf16_bits"](x.astype(np.float64))
+
+
 def _closed_form_wrong(N, k, B):
     return N * (1.0 - (1.0 - k / N) ** (B - 1))
 
@@ -215,6 +229,9 @@ MUTATIONS = {
     "threshold loop runs while f <= target": ("greedy_select_threshold", _threshold_non_strict),
     "threshold ignores the warm-up mass": ("greedy_select_threshold", _threshold_ignores_s0_mass),
     "expert sum left to right": ("expert_tree_sum", _tree_sum_left_to_right),
+    "budget split drops the remainder": ("layer_budgets", _budgets_floor),
+    "bf16 by truncation": ("f64_to_bf16_bits", _bf16_truncate),
+    "bf16 rounded through fp32": ("f64_to_bf16_bits", _bf16_via_fp32),
 }
 
 _orig = {name: getattr(O, name) for name, _ in MUTATIONS.values()}
