@@ -66,6 +66,12 @@ def parse_args(argv=None):
     ap.add_argument("--tau", type=float, default=None, help="covered score-mass fraction (thresh)")
     ap.add_argument("--shared", type=int, default=0,
                     help="shared experts added to every token (DeepSeek-R1 has one)")
+    ap.add_argument("--layers", type=int, default=1,
+                    help="time a stack of this many residual layers, replayed from a CUDA graph")
+    ap.add_argument("--weight-sets", type=int, default=2,
+                    help="distinct expert-weight sets the stack's layers cycle through")
+    ap.add_argument("--global-budget", type=int, default=None,
+                    help="stack budget K (default: layers x the per-layer budget)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--seed", type=int, default=0)
     return ap.parse_args(argv)
@@ -437,6 +443,122 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
     return out
 
 
+def run_gpu_stack(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
+    """L residual layers (xshare_stack_graph_*): one step = one graph replay."""
+    from paper_2602_07265_gb300 import _build
+    _build.build()
+    from paper_2602_07265_gb300 import xshare as X
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    init_dist(world, "nccl")
+    stream = torch.cuda.current_stream()
+    L, P = args.layers, max(1, min(args.weight_sets, args.layers))
+    K_total = args.global_budget if args.global_budget is not None else L * w.budget
+    Ns = args.shared
+    sets = [W.expert_weights(w, args.seed + 10 * s, device=str(dev), down_std=W.STACK_DOWN_STD)
+            for s in range(P)]
+    shared = [W.shared_expert_weights(w, Ns, args.seed + 10 * s, device=str(dev),
+                                      down_std=W.STACK_DOWN_STD) if Ns else None
+              for s in range(P)]
+    layers = []
+    for l in range(L):
+        _, W_g = W.router_inputs(w, args.seed + 1000 + l)
+        layers.append((W_g.to(dev),) + tuple(sets[l % P]) + (shared[l % P],))
+    x_host = W.router_inputs(w, args.seed + 101 * rank)[0]
+    x = x_host.to(dev)
+    prm = X.route_params(**w.params())
+    ws = torch.empty(X.xshare_workspace_size(w.B, w.N, w.k, w.d, w.F, w.mode, prm, Ns),
+                     dtype=torch.uint8, device=dev)
+    h = torch.empty(L, w.B, w.d, dtype=torch.bfloat16, device=dev)
+    st = torch.zeros(L, X.STATS_WORDS, dtype=torch.int32, device=dev)
+    g = X.StackGraph(x, layers, w.k, K_total, w.mode, prm, h, ws, stats=st)
+    K, Wm = args.steps, args.warmup
+    for _ in range(Wm):
+        g.launch(stream)
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize()
+    with sampler:
+        t0.record(stream)
+        for _ in range(K):
+            g.launch(stream)
+        t1.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    ms_total = reduce_max(t0.elapsed_time(t1), world, dev)
+    s = st.cpu().numpy()
+    if np.any(s[:, 5] != 0):
+        raise RuntimeError(f"device status {s[:, 5].max()} (a bounded wait ran out)")
+    n_used, n_pairs = s[:, 1], s[:, 4]
+    ab = [algorithmic_bytes(w, int(n_used[l]), int(n_pairs[l]), Ns) for l in range(L)]
+    stack_bytes = float(sum(a["layer"] for a in ab))
+    flops = float(sum(6 * w.d * w.F * (n_pairs[l] + Ns * w.B) + 2 * w.B * w.N * w.d
+                      for l in range(L)))
+    peaks = measured_peaks()
+    step_s = ms_total / K * 1e-3
+    t_roof = max(stack_bytes / (peaks["hbm_gbs"] * 1e9), flops / (peaks["bf16_tflops"] * 1e12))
+    tokens_total = reduce_sum(w.B * K, world, dev)
+
+    # end to end: x from pinned host memory in, the last layer's output out, every step
+    x_pin = x_host.pin_memory()
+    y_pin = torch.empty(w.B, w.d, dtype=torch.bfloat16).pin_memory()
+
+    def e2e_step():
+        x.copy_(x_pin, non_blocking=True)
+        g.launch(stream)
+        y_pin.copy_(h[L - 1], non_blocking=True)
+        stream.synchronize()
+
+    for _ in range(Wm):
+        e2e_step()
+    barrier(world)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(K):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    e2e_ms = reduce_max(e0.elapsed_time(e1), world, dev)
+    g.close()
+    launches_per_layer = X.N_STAGES - (1 if (w.B + 31) // 32 <= 2 else 0)
+    achieved = stack_bytes / step_s / 1e9
+    return {
+        "metric": METRIC,
+        "value": tokens_total / (ms_total * 1e-3),
+        "unit": "tokens/s",
+        "n_gpus": world, "steps": K, "warmup": Wm,
+        "ms_per_step": ms_total / K,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic",
+        "config": {
+            "workload": f"{describe(w, Ns)}; stack of {L} residual layers (x + MoE(x)), "
+                        f"global budget K={K_total} (m_l = K/L), {P} expert-weight sets, "
+                        "one CUDA-graph replay per step",
+            "B": w.B, "N": w.N, "k": w.k, "d": w.d, "F": w.F, "layers": L, "weight_sets": P,
+            "global_budget": K_total, "shared_experts": Ns, "global_batch": w.B * world,
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+            "l2": f"inputs larger than L2: ~{stack_bytes / 1e9:.1f} GB of expert weights per step",
+        },
+        "experts": {"selected_per_layer": [int(v) for v in s[:, 0]],
+                    "used_per_layer": [int(v) for v in n_used],
+                    "union_topk_per_layer": [int(v) for v in s[:, 2]]},
+        "layer": {"roofline_frac": t_roof / step_s, "algorithmic_gbs": achieved,
+                  "peak_source": peaks["source"]},
+        "roofline": {"kernel": "stack (whole graph replay)", "bound": "hbm", "achieved": achieved,
+                     "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
+                     "traffic": None},
+        "clocks": sampler.summary(),
+        "e2e": {"value": tokens_total / (e2e_ms * 1e-3), "unit": "tokens/s",
+                "h2d_bytes_per_step": w.B * w.d * 2, "d2h_bytes_per_step": w.B * w.d * 2},
+        "gpu_launches": launches_per_layer * L * K,
+    }
+
+
 # --------------------------------------------------------------------------- oracle timing
 
 class OracleSampler:
@@ -561,6 +683,13 @@ def main(argv=None):
         if rank != 0:
             return 0
         print(json.dumps(run_reference(args, w, rank, world)))
+        return 0
+    if args.layers > 1:
+        out = run_gpu_stack(args, w, rank, world, local)
+        if rank == 0:
+            print(json.dumps(out))
+        if world > 1:
+            torch.distributed.destroy_process_group()
         return 0
     out = run_gpu(args, w, rank, world, local)
     if rank == 0:

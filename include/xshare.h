@@ -228,6 +228,65 @@ int xshare_moe_forward_profiled(const uint16_t *x, const float *W_g, const uint1
 /* Name of stage i of xshare_moe_forward (e.g. "router"), or "" if out of range. */
 const char *xshare_stage_name(int i);
 
+/* One MoE layer of a stack: router W_g [N, d] fp32, experts as in
+ * xshare_moe_forward, optional shared experts (NULL: none).  Device pointers;
+ * several layers may point to the same weights. */
+typedef struct {
+  const float *W_g;
+  const uint16_t *W_gate;
+  const uint16_t *W_up;
+  const uint16_t *W_down;
+  const xs_shared_experts *shared;
+} xs_layer;
+
+/* A stack of L MoE layers under one global expert budget (Eq. 1 at the system
+ * level; the paper's practical per-layer budget m_l = K / L, Sec. 3.2):
+ *
+ *   x_{l+1} = x_l + MoE_l(x_l),   l = 0 .. L-1,   x_0 = x,
+ *
+ * where MoE_l is xshare_moe_forward with layer l's weights and selection
+ * budget m_l = floor(K_total / L) + (l < K_total mod L ? 1 : 0), so that the
+ * budgets sum to K_total (used by BATCH and HIER; the other modes take no
+ * budget).  The sum x_l + MoE_l(x_l) is accumulated in fp32 (x_l first) and
+ * rounded once to bf16.
+ *
+ *   x      [B, d] bf16, device: the input of layer 0.
+ *   layers host array of L xs_layer (1 <= L <= 4096).
+ *   h_out  [L, B, d] bf16, device, out: h_out[l] = x_{l+1}; must not overlap x.
+ *   stats  [L] xs_stats, device, out, nullable: layer l's statistics.
+ *   workspace: xshare_workspace_size(B, N, k, d, F, mode, prm, n) bytes with n
+ *          the largest shared-expert count of the layers; the layers run one
+ *          after another on `stream` and reuse it.
+ * Every layer's arguments are checked before the first launch.  The call
+ * launches 6 or 7 kernels per layer and may be captured into a CUDA graph by
+ * the caller; xshare_stack_graph_create does that itself. */
+int xshare_stack_forward(const uint16_t *x, const xs_layer *layers, int L, int B, int d, int F,
+                         int N, int k, int K_total, int mode, const xs_route_params *prm,
+                         uint16_t *h_out, xs_stats *stats, void *workspace, size_t ws_bytes,
+                         xs_stream_t stream);
+
+/* A CUDA graph of one xshare_stack_forward call (opaque). */
+typedef struct xs_graph xs_graph;
+
+/* Captures xshare_stack_forward with these arguments into a CUDA graph on a
+ * private stream and instantiates it; *out receives the handle (NULL on
+ * error).  Nothing runs on the GPU.  The graph keeps every device pointer and
+ * the host values of `layers`, `prm` and the shared-expert descriptors as
+ * they are now: replays read and write the same buffers, which must stay
+ * allocated until xshare_stack_graph_destroy.  CUDA allocates host and device
+ * resources for the graph itself. */
+int xshare_stack_graph_create(const uint16_t *x, const xs_layer *layers, int L, int B, int d,
+                              int F, int N, int k, int K_total, int mode,
+                              const xs_route_params *prm, uint16_t *h_out, xs_stats *stats,
+                              void *workspace, size_t ws_bytes, xs_graph **out);
+
+/* Replays the graph on `stream` (asynchronous).  Replays that share a
+ * workspace or outputs must not overlap. */
+int xshare_stack_graph_launch(xs_graph *g, xs_stream_t stream);
+
+/* Releases the graph (NULL is ignored).  No replay may be pending. */
+void xshare_stack_graph_destroy(xs_graph *g);
+
 /* Self-test of the library's failure reporting (no counterpart in the paper).
  * Launches one kernel that waits, through the same bounded wait every
  * pipeline wait of the library uses, on a barrier that nothing arrives at.

@@ -190,20 +190,20 @@ namespace {
 const char *const kStageNames[XS_N_STAGES] = {"router", "select", "refine", "gather", "ffn_gate_up",
                                               "ffn_down", "combine"};
 
-int forward_impl(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
-                 const uint16_t *W_up, const uint16_t *W_down, int B, int d, int F, int N, int k,
-                 int budget, int mode, const xs_route_params *prm,
-                 const xs_shared_experts *shared, uint16_t *y, float *scores_out,
-                 uint8_t *sel_mask, int32_t *topk_ids, float *topk_w, xs_stats *stats,
-                 void *workspace, size_t ws_bytes, xs_stream_t stream, void *const *events) {
-  int rc = check_route_args(B, N, k, budget, mode, prm);
+}  // namespace
+
+int xs::forward_impl(const FwdCall &c, FwdStep step) {
+  const int B = c.B, d = c.d, F = c.F, N = c.N, k = c.k;
+  int rc = check_route_args(B, N, k, c.budget, c.mode, c.prm);
   if (rc != XS_OK) return rc;
   rc = check_ffn_shape(d, F);
   if (rc != XS_OK) return rc;
-  if (!x || !W_g || !W_gate || !W_up || !W_down || !y) return XS_ERR_NULL;
-  if (!aligned16(x) || !aligned16(W_g) || !aligned16(W_gate) || !aligned16(W_up) ||
-      !aligned16(W_down) || !aligned16(y) || (scores_out && !aligned16(scores_out)))
+  if (!c.x || !c.W_g || !c.W_gate || !c.W_up || !c.W_down || !c.y) return XS_ERR_NULL;
+  if (!aligned16(c.x) || !aligned16(c.W_g) || !aligned16(c.W_gate) || !aligned16(c.W_up) ||
+      !aligned16(c.W_down) || !aligned16(c.y) || (c.scores_out && !aligned16(c.scores_out)) ||
+      (c.resid && !aligned16(c.resid)))
     return XS_ERR_ALIGN;
+  const xs_shared_experts *shared = c.shared;
   const int n_shared = shared ? shared->n_shared : 0;
   if (n_shared < 0 || n_shared > kMaxShared) return XS_ERR_PARAM;
   if (n_shared > 0) {
@@ -211,30 +211,34 @@ int forward_impl(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
     if (!aligned16(shared->W_gate) || !aligned16(shared->W_up) || !aligned16(shared->W_down))
       return XS_ERR_ALIGN;
   }
+  void *workspace = c.workspace;
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return XS_ERR_WORKSPACE;
+  if (step == FwdStep::kCheckArgs) return XS_OK;
   const int sms = current_device_sms();
   if (sms < 0) return sms;
   const Plan pl = make_plan(B, N, k, d, F, true, sms, n_shared);
-  if (ws_bytes < pl.total) return XS_ERR_WORKSPACE;
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (c.ws_bytes < pl.total) return XS_ERR_WORKSPACE;
+  if (step == FwdStep::kCheckAll) return XS_OK;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(c.stream);
+  void *const *events = c.events;
 
-  RouteArgs a = route_args(pl, workspace, B, N, k, budget, mode, prm);
+  RouteArgs a = route_args(pl, workspace, B, N, k, c.budget, c.mode, c.prm);
   float *h = at<float>(workspace, pl.h);
   a.logits = h;
-  if (scores_out) a.p = scores_out;
-  if (sel_mask) a.mask = sel_mask;
-  if (topk_ids) a.ids = topk_ids;
-  if (topk_w) a.w = topk_w;
-  a.stats = stats;
+  if (c.scores_out) a.p = c.scores_out;
+  if (c.sel_mask) a.mask = c.sel_mask;
+  if (c.topk_ids) a.ids = c.topk_ids;
+  if (c.topk_w) a.w = c.topk_w;
+  a.stats = c.stats;
   a.zero_words = at<int32_t>(workspace, pl.ffn_cnt);
   a.zero_count = (int)ffn_cnt_words(pl.max_tiles, B, d, F);
   a.n_shared = n_shared;
 
   FfnArgs f;
   std::memset(&f, 0, sizeof(f));
-  f.W_gate = W_gate;
-  f.W_up = W_up;
-  f.W_down = W_down;
+  f.W_gate = c.W_gate;
+  f.W_up = c.W_up;
+  f.W_down = c.W_down;
   if (n_shared > 0) {
     f.S_gate = shared->W_gate;
     f.S_up = shared->W_up;
@@ -246,7 +250,7 @@ int forward_impl(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
   f.out = at<float>(workspace, pl.out);
   f.tiles = a.tiles;
   f.meta = a.meta;
-  f.stats = stats;
+  f.stats = c.stats;
   f.part = at<void>(workspace, pl.ffn_part);
   f.cnt = at<int32_t>(workspace, pl.ffn_cnt);
   f.N = N;
@@ -261,20 +265,58 @@ int forward_impl(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
            cudaEventRecord(reinterpret_cast<cudaEvent_t>(events[i]), s) == cudaSuccess;
   };
   if (!mark(0)) return XS_ERR_CUDA;
-  if (launch_router_logits(x, W_g, h, B, N, d, a.done, s) != cudaSuccess || !mark(1))
+  if (launch_router_logits(c.x, c.W_g, h, B, N, d, a.done, s) != cudaSuccess || !mark(1))
     return XS_ERR_CUDA;
   a.events = events ? events + 2 : nullptr;  // between the selection and refinement kernels
   if (launch_route(a, s) != cudaSuccess || !mark(3)) return XS_ERR_CUDA;
-  if (launch_gather(x, a.perm, a.meta, const_cast<uint16_t *>(f.xp), pl.max_rows, B, d, k, s) !=
-          cudaSuccess ||
+  if (launch_gather(c.x, a.perm, a.meta, const_cast<uint16_t *>(f.xp), pl.max_rows, B, d, k,
+                    s) != cudaSuccess ||
       !mark(4))
     return XS_ERR_CUDA;
   if (launch_ffn_gate_up(f, s) != cudaSuccess || !mark(5)) return XS_ERR_CUDA;
   if (launch_ffn_down(f, s) != cudaSuccess || !mark(6)) return XS_ERR_CUDA;
-  if (launch_combine(f.out, a.pos, a.w, a.meta, y, B, d, k, n_shared, s) != cudaSuccess ||
+  if (launch_combine(f.out, a.pos, a.w, a.meta, c.resid, c.y, B, d, k, n_shared, s) !=
+          cudaSuccess ||
       !mark(7))
     return XS_ERR_CUDA;
   return XS_OK;
+}
+
+namespace {
+
+FwdCall make_call(const uint16_t *x, const float *W_g, const uint16_t *W_gate,
+                  const uint16_t *W_up, const uint16_t *W_down, int B, int d, int F, int N, int k,
+                  int budget, int mode, const xs_route_params *prm, const xs_shared_experts *shared,
+                  uint16_t *y, float *scores_out, uint8_t *sel_mask, int32_t *topk_ids,
+                  float *topk_w, xs_stats *stats, void *workspace, size_t ws_bytes,
+                  xs_stream_t stream, void *const *events) {
+  FwdCall c;
+  std::memset(&c, 0, sizeof(c));
+  c.x = x;
+  c.W_g = W_g;
+  c.W_gate = W_gate;
+  c.W_up = W_up;
+  c.W_down = W_down;
+  c.B = B;
+  c.d = d;
+  c.F = F;
+  c.N = N;
+  c.k = k;
+  c.budget = budget;
+  c.mode = mode;
+  c.prm = prm;
+  c.shared = shared;
+  c.y = y;
+  c.scores_out = scores_out;
+  c.sel_mask = sel_mask;
+  c.topk_ids = topk_ids;
+  c.topk_w = topk_w;
+  c.stats = stats;
+  c.workspace = workspace;
+  c.ws_bytes = ws_bytes;
+  c.stream = stream;
+  c.events = events;
+  return c;
 }
 
 }  // namespace
@@ -286,9 +328,10 @@ extern "C" int xshare_moe_forward(const uint16_t *x, const float *W_g, const uin
                                   uint16_t *y, float *scores_out, uint8_t *sel_mask,
                                   int32_t *topk_ids, float *topk_w, xs_stats *stats,
                                   void *workspace, size_t ws_bytes, xs_stream_t stream) {
-  return forward_impl(x, W_g, W_gate, W_up, W_down, B, d, F, N, k, budget, mode, prm, shared, y,
-                      scores_out, sel_mask, topk_ids, topk_w, stats, workspace, ws_bytes, stream,
-                      nullptr);
+  return forward_impl(make_call(x, W_g, W_gate, W_up, W_down, B, d, F, N, k, budget, mode, prm,
+                                shared, y, scores_out, sel_mask, topk_ids, topk_w, stats,
+                                workspace, ws_bytes, stream, nullptr),
+                      FwdStep::kLaunch);
 }
 
 extern "C" int xshare_moe_forward_profiled(const uint16_t *x, const float *W_g,
@@ -304,9 +347,10 @@ extern "C" int xshare_moe_forward_profiled(const uint16_t *x, const float *W_g,
   if (stage_events == nullptr) return XS_ERR_NULL;
   for (int i = 0; i <= XS_N_STAGES; ++i)
     if (stage_events[i] == nullptr) return XS_ERR_NULL;
-  return forward_impl(x, W_g, W_gate, W_up, W_down, B, d, F, N, k, budget, mode, prm, shared, y,
-                      scores_out, sel_mask, topk_ids, topk_w, stats, workspace, ws_bytes, stream,
-                      stage_events);
+  return forward_impl(make_call(x, W_g, W_gate, W_up, W_down, B, d, F, N, k, budget, mode, prm,
+                                shared, y, scores_out, sel_mask, topk_ids, topk_w, stats,
+                                workspace, ws_bytes, stream, stage_events),
+                      FwdStep::kLaunch);
 }
 
 extern "C" const char *xshare_stage_name(int i) {

@@ -879,12 +879,14 @@ __global__ void __launch_bounds__(256) gather_kernel(const uint16_t *__restrict_
   for (int i = threadIdx.x; i < d / 8; i += blockDim.x) dst[i] = __ldg(src + i);
 }
 
-// ---- a9: y_t = sum over slots s < k' of w_ts * out[pos(t, s)]
+// ---- a9: y_t = [x_t +] sum over slots s < k' of w_ts * out[pos(t, s)]
 //              + sum over shared experts j of out[n_pairs + j * B + t], fp32, bf16 once.
+// The residual x_t is added first when `resid` is given (layer stacks).
 __global__ void __launch_bounds__(256) combine_kernel(const float *__restrict__ out,
                                                       const int32_t *__restrict__ pos,
                                                       const float *__restrict__ w,
                                                       const Meta *__restrict__ meta,
+                                                      const uint16_t *__restrict__ resid,
                                                       uint16_t *__restrict__ y, int B, int d,
                                                       int k, int n_shared) {
   pdl_wait();
@@ -894,6 +896,13 @@ __global__ void __launch_bounds__(256) combine_kernel(const float *__restrict__ 
   if (c4 >= d / 4) return;
   const int kp = meta->kprime;
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (resid != nullptr) {
+    const uint2 r = reinterpret_cast<const uint2 *>(resid + (size_t)t * d)[c4];
+    acc.x = __uint_as_float(r.x << 16);
+    acc.y = __uint_as_float(r.x & 0xffff0000u);
+    acc.z = __uint_as_float(r.y << 16);
+    acc.w = __uint_as_float(r.y & 0xffff0000u);
+  }
   for (int s = 0; s < kp; ++s) {
     const int r = pos[(size_t)t * k + s];
     if (r < 0) continue;  // only with non-finite scores
@@ -967,10 +976,10 @@ cudaError_t launch_gather(const uint16_t *x, const int32_t *perm, const Meta *me
 }
 
 cudaError_t launch_combine(const float *out, const int32_t *pos, const float *w,
-                           const Meta *meta, uint16_t *y, int B, int d, int k, int n_shared,
-                           cudaStream_t s) {
+                           const Meta *meta, const uint16_t *resid, uint16_t *y, int B, int d,
+                           int k, int n_shared, cudaStream_t s) {
   dim3 grid((d / 4 + 255) / 256, B);
-  return launch_pdl(combine_kernel, grid, dim3(256), 0, s, out, pos, w, meta, y, B, d, k,
+  return launch_pdl(combine_kernel, grid, dim3(256), 0, s, out, pos, w, meta, resid, y, B, d, k,
                     n_shared);
 }
 

@@ -120,8 +120,8 @@ cudaError_t launch_route(const RouteArgs &a, cudaStream_t s);
 cudaError_t launch_router_logits(const uint16_t *x, const float *Wg, float *h, int B, int N,
                                  int d, int32_t *done, cudaStream_t s);
 cudaError_t launch_combine(const float *out, const int32_t *pos, const float *w,
-                           const Meta *meta, uint16_t *y, int B, int d, int k, int n_shared,
-                           cudaStream_t s);
+                           const Meta *meta, const uint16_t *resid, uint16_t *y, int B, int d,
+                           int k, int n_shared, cudaStream_t s);
 cudaError_t launch_gather(const uint16_t *x, const int32_t *perm, const Meta *meta,
                           uint16_t *xp, int max_rows, int B, int d, int k, cudaStream_t s);
 
@@ -144,5 +144,34 @@ cudaError_t launch_ffn_gate_up(const FfnArgs &a, cudaStream_t s);
 cudaError_t launch_ffn_down(const FfnArgs &a, cudaStream_t s);
 size_t ffn_part_bytes(int n_sms);
 size_t ffn_cnt_words(int max_tiles, int B, int d, int F);
+
+// One MoE-layer forward as the C entry points describe it, plus `resid`
+// (nullable): x_t added to y_t before rounding.
+struct FwdCall {
+  const uint16_t *x;
+  const float *W_g;
+  const uint16_t *W_gate, *W_up, *W_down;
+  int B, d, F, N, k, budget, mode;
+  const xs_route_params *prm;
+  const xs_shared_experts *shared;
+  const uint16_t *resid;
+  uint16_t *y;
+  float *scores_out;
+  uint8_t *sel_mask;
+  int32_t *topk_ids;
+  float *topk_w;
+  xs_stats *stats;
+  void *workspace;
+  size_t ws_bytes;
+  xs_stream_t stream;
+  void *const *events;
+};
+
+enum class FwdStep {
+  kCheckArgs,   // host-side argument checks only (no CUDA call)
+  kCheckAll,    // also the device and the workspace size
+  kLaunch,      // check everything, then launch
+};
+int forward_impl(const FwdCall &c, FwdStep step);
 
 }  // namespace xs

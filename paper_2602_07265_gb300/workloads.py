@@ -30,6 +30,13 @@ MODES = {"topk": MODE_TOPK, "batch": MODE_BATCH, "group": MODE_GROUP, "hier": MO
          "thresh": MODE_THRESH}
 
 EXPERT_STD = 0.02
+# Layer stacks add each layer's output to the residual stream x.  A SwiGLU
+# expert's output grows with |x|^2, so at N(0, 0.02) a DeepSeek-R1-sized layer
+# returns about |x| itself and a stack's activations explode within a few
+# layers.  Stacks therefore draw W_down with a ten times smaller deviation:
+# a layer then adds roughly a tenth of |x|, and |x| stays near 1 over tens of
+# layers (there is no normalisation between layers).
+STACK_DOWN_STD = 0.002
 
 
 @dataclasses.dataclass(frozen=True)
@@ -127,9 +134,10 @@ def batch_stream(w: Workload, seed: int, count: int) -> list:
 
 
 def expert_weights(w: Workload, seed: int = 0, device: str = "cuda",
-                   experts: Optional[list] = None,
-                   f_rows: Optional[int] = None) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
-    """W_gate [N, F, d], W_up [N, F, d], W_down [N, d, F], bf16, N(0, 0.02).
+                   experts: Optional[list] = None, f_rows: Optional[int] = None,
+                   down_std: float = EXPERT_STD) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    """W_gate [N, F, d], W_up [N, F, d], W_down [N, d, F], bf16, N(0, 0.02)
+    (W_down N(0, down_std)).
 
     Drawn expert by expert from a generator on `device`, so that peak
     temporary memory stays at one fp32 expert matrix.  With `experts` given
@@ -148,22 +156,26 @@ def expert_weights(w: Workload, seed: int = 0, device: str = "cuda",
     if device == "cpu" or experts is not None or f_rows is not None:
         for i, e in enumerate(ids):
             g = _gen(seed, 1000 + e)
-            for t, shape in ((Wg, (F, d)), (Wu, (F, d)), (Wd, (d, F))):
-                t[i].copy_(torch.randn(*shape, generator=g) * EXPERT_STD)
+            for t, shape, std in ((Wg, (F, d), EXPERT_STD), (Wu, (F, d), EXPERT_STD),
+                                  (Wd, (d, F), down_std)):
+                t[i].copy_(torch.randn(*shape, generator=g) * std)
     else:
         g = torch.Generator(device=device)
         g.manual_seed(int(seed) * 1_000_003 + 7)
         for i in range(n):
-            for t, shape in ((Wg, (F, d)), (Wu, (F, d)), (Wd, (d, F))):
-                t[i].copy_(torch.randn(*shape, generator=g, device=device) * EXPERT_STD)
+            for t, shape, std in ((Wg, (F, d), EXPERT_STD), (Wu, (F, d), EXPERT_STD),
+                                  (Wd, (d, F), down_std)):
+                t[i].copy_(torch.randn(*shape, generator=g, device=device) * std)
     return Wg, Wu, Wd
 
 
-def shared_expert_weights(w: Workload, n_shared: int, seed: int = 0,
-                          device: str = "cuda") -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+def shared_expert_weights(w: Workload, n_shared: int, seed: int = 0, device: str = "cuda",
+                          down_std: float = EXPERT_STD
+                          ) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
     """Shared experts [n_shared, F, d], [n_shared, F, d], [n_shared, d, F], bf16,
-    N(0, 0.02), from a seed stream apart from the routed experts'."""
-    return expert_weights(w.with_(N=n_shared), seed + 7_777_777, device=device)
+    N(0, 0.02) (W_down N(0, down_std)), from a seed stream apart from the
+    routed experts'."""
+    return expert_weights(w.with_(N=n_shared), seed + 7_777_777, device=device, down_std=down_std)
 
 
 def random_scores(B: int, N: int, seed: int, ties: bool = False) -> np.ndarray:

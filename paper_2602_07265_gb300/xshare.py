@@ -47,6 +47,13 @@ class SharedExperts(ctypes.Structure):
 MAX_SHARED = 8
 
 
+class Layer(ctypes.Structure):
+    """xs_layer (device pointers; `shared` points to an SharedExperts or is NULL)."""
+    _fields_ = [("W_g", ctypes.c_void_p), ("W_gate", ctypes.c_void_p),
+                ("W_up", ctypes.c_void_p), ("W_down", ctypes.c_void_p),
+                ("shared", ctypes.POINTER(SharedExperts))]
+
+
 def route_params(k0: int = 0, m_r: int = 0, tokens_per_request: int = 1, n_groups: int = 1,
                  m_g: int = 0, tau: float = 0.0) -> RouteParams:
     return RouteParams(k0, m_r, tokens_per_request, n_groups, m_g, tau)
@@ -72,6 +79,16 @@ def _load() -> ctypes.CDLL:
     lib.xshare_route_static.restype = I
     lib.xshare_moe_forward_profiled.argtypes = lib.xshare_moe_forward.argtypes + [P]
     lib.xshare_moe_forward_profiled.restype = I
+    PL = ctypes.POINTER(Layer)
+    lib.xshare_stack_forward.argtypes = [P, PL, I, I, I, I, I, I, I, I, PR, P, P, P, Z, P]
+    lib.xshare_stack_forward.restype = I
+    lib.xshare_stack_graph_create.argtypes = [P, PL, I, I, I, I, I, I, I, I, PR, P, P, P, Z,
+                                              ctypes.POINTER(P)]
+    lib.xshare_stack_graph_create.restype = I
+    lib.xshare_stack_graph_launch.argtypes = [P, P]
+    lib.xshare_stack_graph_launch.restype = I
+    lib.xshare_stack_graph_destroy.argtypes = [P]
+    lib.xshare_stack_graph_destroy.restype = None
     lib.xshare_selftest_wait_timeout.argtypes = [P, ctypes.c_uint64, P]
     lib.xshare_selftest_wait_timeout.restype = I
     lib.xshare_stage_name.argtypes = [I]
@@ -217,6 +234,77 @@ def xshare_moe_forward(x: torch.Tensor, W_g: torch.Tensor, W_gate: torch.Tensor,
             ev.record()   # torch creates the CUDA event lazily
         handles[i] = ev.cuda_event
     _check(LIB.xshare_moe_forward_profiled(*args, handles), "xshare_moe_forward_profiled")
+
+
+def _stack_args(x, layers, k, K_total, mode, params, h_out, workspace, stats):
+    """Marshals a layer stack: `layers` is a list of (W_g, W_gate, W_up, W_down)
+    or (W_g, W_gate, W_up, W_down, (S_gate, S_up, S_down)) tensors."""
+    B, d = x.shape
+    L = len(layers)
+    if L < 1:
+        raise ValueError("at least one layer")
+    N, F = layers[0][1].shape[0], layers[0][1].shape[1]
+    arr = (Layer * L)()
+    keep = []
+    for l, lay in enumerate(layers):
+        W_g, Wg, Wu, Wd = lay[:4]
+        if W_g.shape != (N, d) or tuple(Wg.shape) != (N, F, d) or tuple(Wu.shape) != (N, F, d) \
+                or tuple(Wd.shape) != (N, d, F):
+            raise ValueError(f"layer {l}: inconsistent shapes")
+        arr[l].W_g = _ptr(W_g, torch.float32, "W_g")
+        arr[l].W_gate = _ptr(Wg, torch.bfloat16, "W_gate")
+        arr[l].W_up = _ptr(Wu, torch.bfloat16, "W_up")
+        arr[l].W_down = _ptr(Wd, torch.bfloat16, "W_down")
+        if len(lay) > 4 and lay[4] is not None:
+            Sg, Su, Sd = lay[4]
+            sh = SharedExperts(_ptr(Sg, torch.bfloat16, "S_gate"), _ptr(Su, torch.bfloat16, "S_up"),
+                               _ptr(Sd, torch.bfloat16, "S_down"), Sg.shape[0])
+            keep.append(sh)
+            arr[l].shared = ctypes.pointer(sh)
+    if tuple(h_out.shape) != (L, B, d):
+        raise ValueError("h_out must be [L, B, d]")
+    args = [_ptr(x, torch.bfloat16, "x"), arr, L, B, d, F, N, k, K_total, mode,
+            ctypes.byref(params), _ptr(h_out, torch.bfloat16, "h_out"),
+            _ptr(stats, torch.int32, "stats", L * STATS_WORDS),
+            _ptr(workspace, torch.uint8, "workspace"), workspace.numel()]
+    return args, keep
+
+
+def xshare_stack_forward(x: torch.Tensor, layers: list, k: int, K_total: int, mode: int,
+                         params: RouteParams, h_out: torch.Tensor, workspace: torch.Tensor,
+                         stats: Optional[torch.Tensor] = None, stream=None) -> None:
+    """L residual MoE layers under the global budget K_total into h_out [L, B, d]; see xshare.h."""
+    args, keep = _stack_args(x, layers, k, K_total, mode, params, h_out, workspace, stats)
+    _check(LIB.xshare_stack_forward(*args, _stream(stream)), "xshare_stack_forward")
+    del keep
+
+
+class StackGraph:
+    """xshare_stack_graph_create / _launch / _destroy.  Keeps references to the
+    tensors it was captured with, which replays read and write."""
+
+    def __init__(self, x, layers, k, K_total, mode, params, h_out, workspace, stats=None):
+        self._args, self._keep = _stack_args(x, layers, k, K_total, mode, params, h_out,
+                                             workspace, stats)
+        self._tensors = (x, layers, h_out, workspace, stats, params)
+        self._handle = ctypes.c_void_p()
+        _check(LIB.xshare_stack_graph_create(*self._args, ctypes.byref(self._handle)),
+               "xshare_stack_graph_create")
+
+    def launch(self, stream=None) -> None:
+        _check(LIB.xshare_stack_graph_launch(self._handle, _stream(stream)),
+               "xshare_stack_graph_launch")
+
+    def close(self) -> None:
+        if self._handle:
+            LIB.xshare_stack_graph_destroy(self._handle)
+            self._handle = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:  # noqa: BLE001 - interpreter shutdown
+            pass
 
 
 def xshare_selftest_wait_timeout(stats: torch.Tensor, budget_ns: int, stream=None) -> None:

@@ -29,7 +29,9 @@ def declared_functions():
 def test_header_declares_the_boundary():
     assert declared_functions() == ["xshare_moe_forward", "xshare_moe_forward_profiled",
                                     "xshare_route", "xshare_route_static",
-                                    "xshare_selftest_wait_timeout", "xshare_stage_name",
+                                    "xshare_selftest_wait_timeout", "xshare_stack_forward",
+                                    "xshare_stack_graph_create", "xshare_stack_graph_destroy",
+                                    "xshare_stack_graph_launch", "xshare_stage_name",
                                     "xshare_strerror",
                                     "xshare_workspace_size"]
 
@@ -112,3 +114,30 @@ def test_workspace_size_rejects_invalid(X):
     assert X.xshare_workspace_size(8, 16, 4, 100, 256, 1, prm) == 0
     assert X.xshare_workspace_size(8, 16, 4, 256, 256, 1, prm, 9) == 0
     assert X.xshare_workspace_size(8, 16, 4, 0, 0, 1, prm, 1) == 0  # routing alone has none
+
+
+def test_stack_rejects_bad_arguments(X):
+    prm = X.route_params()
+    P = 1 << 20
+    lay = (X.Layer * 2)()
+    for l in range(2):
+        lay[l].W_g = lay[l].W_gate = lay[l].W_up = lay[l].W_down = P
+    def rc(L=2, x=P, h=P << 4, d=256, F=256, K=8, layers=lay):
+        return X.LIB.xshare_stack_forward(x, layers, L, 4, d, F, 16, 2, K, 1, ctypes.byref(prm),
+                                          h, None, P, 1 << 20, None)
+    assert rc(L=0) == -1
+    assert rc(K=-1) == -2
+    assert rc(x=None) == -3
+    assert rc(layers=None) == -3
+    assert rc(h=P) == -2            # output overlaps the input
+    assert rc(d=100) == -1
+    lay[1].W_up = None               # a later layer is checked before anything runs
+    assert rc() == -3
+    lay[1].W_up = P
+    out = ctypes.c_void_p(7)
+    assert X.LIB.xshare_stack_graph_create(P, lay, 0, 4, 256, 256, 16, 2, 8, 1,
+                                           ctypes.byref(prm), P << 4, None, P, 1 << 20,
+                                           ctypes.byref(out)) == -1
+    assert not out.value
+    assert X.LIB.xshare_stack_graph_launch(None, None) == -3
+    X.LIB.xshare_stack_graph_destroy(None)
