@@ -188,7 +188,20 @@ def warmup_set(p: np.ndarray, k0: int, tokens: Sequence[int]) -> Set[int]:
 # Selection algorithms
 # --------------------------------------------------------------------------
 
-def greedy_select_budget(scores: np.ndarray, m: int, S0: Set[int]) -> Set[int]:
+def candidates(scores: np.ndarray, S: Set[int], positive_only: bool,
+               pool: Optional[Sequence[int]] = None) -> List[int]:
+    """Experts of `pool` (all of E by default) outside S that may be added.
+
+    With `positive_only` (the sparse-score reading of Sec. 2.2, where g is 0
+    outside each token's top-k) an expert whose column score is 0 has no gain
+    and is never added.
+    """
+    pool = range(scores.shape[0]) if pool is None else pool
+    return [e for e in pool if e not in S and (not positive_only or scores[e] > 0)]
+
+
+def greedy_select_budget(scores: np.ndarray, m: int, S0: Set[int],
+                         positive_only: bool = False) -> Set[int]:
     """Algorithm 1 in the fixed-budget form used in practice (Sec. 3.4).
 
     Starting from S_0, repeatedly add argmax_{e in E \\ S} scores[e], m times
@@ -197,10 +210,9 @@ def greedy_select_budget(scores: np.ndarray, m: int, S0: Set[int]) -> Set[int]:
     By Proposition 1 the marginal gain of e is scores[e] whatever S is, so the
     argmax is taken over the precomputed column scores.
     """
-    N = scores.shape[0]
     S = set(S0)
     for _ in range(m):
-        rest = [e for e in range(N) if e not in S]
+        rest = candidates(scores, S, positive_only)
         if not rest:
             break
         S.add(ranked(scores, rest)[0])
@@ -230,7 +242,8 @@ def expert_tree_sum(values: np.ndarray, members: Set[int]) -> np.float32:
     return np.float32(v[0])
 
 
-def greedy_select_threshold(scores: np.ndarray, tau: float, S0: Set[int]) -> Set[int]:
+def greedy_select_threshold(scores: np.ndarray, tau: float, S0: Set[int],
+                            positive_only: bool = False) -> Set[int]:
     """Algorithm 1 as printed, with a threshold tau on the covered score mass.
 
     Starting from S_0, while f(S) < tau * f(E), add argmax_{e in E \\ S}
@@ -248,7 +261,7 @@ def greedy_select_threshold(scores: np.ndarray, tau: float, S0: Set[int]) -> Set
     target = np.float32(np.float32(tau) * expert_tree_sum(scores, set(range(N))))
     f = expert_tree_sum(scores, S)
     while f < target:
-        rest = [e for e in range(N) if e not in S]
+        rest = candidates(scores, S, positive_only)
         if not rest:
             break
         e = ranked(scores, rest)[0]
@@ -257,38 +270,43 @@ def greedy_select_threshold(scores: np.ndarray, tau: float, S0: Set[int]) -> Set
     return S
 
 
-def select_threshold(p: np.ndarray, tau: float, k0: int) -> Tuple[Set[int], Set[int]]:
+def select_threshold(p: np.ndarray, tau: float, k0: int,
+                     gs: Optional[np.ndarray] = None) -> Tuple[Set[int], Set[int]]:
     """Algorithm 2 with GreedySelect in its threshold form: warm-up S_0, then
-    add experts until they cover a fraction tau of the batch's score mass."""
+    add experts until they cover a fraction tau of the batch's score mass.
+    With `gs` (sparse scores) the column scores are taken from gs."""
     B = p.shape[0]
     S0 = warmup_set(p, k0, range(B))
-    scores = canonical_column_sum(p, range(B))
-    return greedy_select_threshold(scores, tau, S0), S0
+    scores = canonical_column_sum(p if gs is None else gs, range(B))
+    return greedy_select_threshold(scores, tau, S0, gs is not None), S0
 
 
-def select_batch(p: np.ndarray, m: int, k0: int) -> Tuple[Set[int], Set[int]]:
-    """Algorithm 2: warm-up S_0, then GreedySelect with budget m.  Returns (S, S_0)."""
+def select_batch(p: np.ndarray, m: int, k0: int,
+                 gs: Optional[np.ndarray] = None) -> Tuple[Set[int], Set[int]]:
+    """Algorithm 2: warm-up S_0, then GreedySelect with budget m.  Returns (S, S_0).
+    With `gs` (sparse scores) the column scores are taken from gs."""
     B = p.shape[0]
     S0 = warmup_set(p, k0, range(B))
-    scores = canonical_column_sum(p, range(B))
-    return greedy_select_budget(scores, m, S0), S0
+    scores = canonical_column_sum(p if gs is None else gs, range(B))
+    return greedy_select_budget(scores, m, S0, gs is not None), S0
 
 
-def per_request_select(p: np.ndarray, tokens: Sequence[int], m_r: int, k0: int) -> Set[int]:
+def per_request_select(p: np.ndarray, tokens: Sequence[int], m_r: int, k0: int,
+                       gs: Optional[np.ndarray] = None) -> Set[int]:
     """Algorithm 3 for one request r with tokens T_r.
 
     S_0 = union of Top k0 over T_r; scores[j] = sum over T_r of g_xj (Eq. 3);
-    S_r = S_0 union Top m_r(scores, E \\ S_0).
+    S_r = S_0 union Top m_r(scores, E \\ S_0).  With `gs` (sparse scores) the
+    request's column scores are taken from gs.
     """
-    N = p.shape[1]
     S0 = warmup_set(p, k0, tokens)
-    scores = canonical_column_sum(p, tokens)
-    rest = [e for e in range(N) if e not in S0]
+    scores = canonical_column_sum(p if gs is None else gs, tokens)
+    rest = candidates(scores, S0, gs is not None)
     return S0 | set(top(scores, m_r, rest))
 
 
-def select_hier(p: np.ndarray, m: int, m_r: int, k0: int,
-                tokens_per_request: int) -> Tuple[Set[int], Set[int]]:
+def select_hier(p: np.ndarray, m: int, m_r: int, k0: int, tokens_per_request: int,
+                gs: Optional[np.ndarray] = None) -> Tuple[Set[int], Set[int]]:
     """Algorithm 4: union of per-request selections, then GreedySelect(m).
 
     Requests are contiguous runs of `tokens_per_request` = 1 + L_s tokens
@@ -298,9 +316,9 @@ def select_hier(p: np.ndarray, m: int, m_r: int, k0: int,
     T = tokens_per_request
     S_b: Set[int] = set()
     for r in range(B // T):
-        S_b |= per_request_select(p, range(r * T, (r + 1) * T), m_r, k0)
-    scores = canonical_column_sum(p, range(B))
-    return greedy_select_budget(scores, m, S_b), S_b
+        S_b |= per_request_select(p, range(r * T, (r + 1) * T), m_r, k0, gs)
+    scores = canonical_column_sum(p if gs is None else gs, range(B))
+    return greedy_select_budget(scores, m, S_b, gs is not None), S_b
 
 
 def group_of(e: int, N: int, G: int) -> int:
@@ -308,7 +326,8 @@ def group_of(e: int, N: int, G: int) -> int:
     return e // (N // G)
 
 
-def gpu_aware_greedy(scores: np.ndarray, G: int, m_g: int, S0: Set[int]) -> Set[int]:
+def gpu_aware_greedy(scores: np.ndarray, G: int, m_g: int, S0: Set[int],
+                     positive_only: bool = False) -> Set[int]:
     """Algorithm 5 taken literally.
 
     S = S_0; while |S| < m_g * G: for g = 1..G: add the argmax of the marginal
@@ -323,7 +342,7 @@ def gpu_aware_greedy(scores: np.ndarray, G: int, m_g: int, S0: Set[int]) -> Set[
     while len(S) < m_g * G:
         added = False
         for g in range(G):
-            rest = [e for e in range(g * size, (g + 1) * size) if e not in S]
+            rest = candidates(scores, S, positive_only, range(g * size, (g + 1) * size))
             if not rest:
                 continue
             S.add(ranked(scores, rest)[0])
@@ -333,12 +352,37 @@ def gpu_aware_greedy(scores: np.ndarray, G: int, m_g: int, S0: Set[int]) -> Set[
     return S
 
 
-def select_group(p: np.ndarray, G: int, m_g: int, k0: int) -> Tuple[Set[int], Set[int]]:
-    """Algorithm 6: warm-up S_0 over the batch, then Algorithm 5.  Returns (S, S_0)."""
+def select_group(p: np.ndarray, G: int, m_g: int, k0: int,
+                 gs: Optional[np.ndarray] = None) -> Tuple[Set[int], Set[int]]:
+    """Algorithm 6: warm-up S_0 over the batch, then Algorithm 5.  Returns (S, S_0).
+    With `gs` (sparse scores) the column scores are taken from gs."""
     B = p.shape[0]
     S0 = warmup_set(p, k0, range(B))
-    scores = canonical_column_sum(p, range(B))
-    return gpu_aware_greedy(scores, G, m_g, S0), S0
+    scores = canonical_column_sum(p if gs is None else gs, range(B))
+    return gpu_aware_greedy(scores, G, m_g, S0, gs is not None), S0
+
+
+def topk_gating(p: np.ndarray, k: int) -> np.ndarray:
+    """Sec. 2.2's gating values: g_ij = exp(h_j) / sum_{T_i} exp(h) for j in
+    T_i = Top k(G_i, E), and 0 outside T_i (the sparse reading of the scores
+    that Sec. 3 sums).
+
+    exp(h_j) / sum_T exp(h) = p_j / sum_T p for the dense softmax p, so each
+    row is computed from p as the standard top-k routing weights are: D = fp32
+    sum of p over T_i in rank order, one fp32 division per expert; if D = 0
+    each of the k experts gets 1/k.  Returns [B, N] float32.
+    """
+    p = np.asarray(p, dtype=np.float32)
+    B, N = p.shape
+    g = np.zeros((B, N), dtype=np.float32)
+    for i in range(B):
+        T = top(p[i], k, range(N))
+        D = np.float32(0.0)
+        for j in T:
+            D = np.float32(D + p[i, j])
+        for j in T:
+            g[i, j] = np.float32(p[i, j] / D) if D > 0 else np.float32(1.0) / np.float32(len(T))
+    return g
 
 
 # --------------------------------------------------------------------------
@@ -416,7 +460,7 @@ def permute(ids: np.ndarray, N: int) -> Dict[str, np.ndarray]:
 
 def route(p: np.ndarray, k: int, budget: int, mode: int, k0: int = 0, m_r: int = 0,
           tokens_per_request: int = 1, n_groups: int = 1, m_g: int = 0,
-          tau: float = 0.0) -> Dict[str, object]:
+          tau: float = 0.0, sparse_scores: int = 0) -> Dict[str, object]:
     """Batch-aware selection and refinement on fp32 gating scores p [B, N].
 
     mode TOPK : S = E (standard top-k routing, the paper's baseline)
@@ -424,21 +468,25 @@ def route(p: np.ndarray, k: int, budget: int, mode: int, k0: int = 0, m_r: int =
     mode HIER : Algorithm 4 with batch budget m = `budget`, per-request m_r, k0
     mode GROUP: Algorithm 6 with G = n_groups contiguous groups, per-group m_g, k0
     mode THRESH: Algorithm 2 with Algorithm 1's threshold tau (fp32), k0; no budget
+    With `sparse_scores` the column scores of every selection step sum Sec.
+    2.2's top-k-masked g instead of the dense softmax, and experts with a zero
+    column score are never added; warm-up and refinement use the dense scores.
     Returns the selected mask, the routing, the permutation and the statistics
     |S|, |U|, |union of plain top-k| and max_g |S intersect E_g|.
     """
     p = np.asarray(p, dtype=np.float32)
     B, N = p.shape
+    gs = topk_gating(p, k) if sparse_scores and mode != MODE_TOPK else None
     if mode == MODE_TOPK:
         S = set(range(N))
     elif mode == MODE_BATCH:
-        S, _ = select_batch(p, budget, k0)
+        S, _ = select_batch(p, budget, k0, gs)
     elif mode == MODE_HIER:
-        S, _ = select_hier(p, budget, m_r, k0, tokens_per_request)
+        S, _ = select_hier(p, budget, m_r, k0, tokens_per_request, gs)
     elif mode == MODE_GROUP:
-        S, _ = select_group(p, n_groups, m_g, k0)
+        S, _ = select_group(p, n_groups, m_g, k0, gs)
     elif mode == MODE_THRESH:
-        S, _ = select_threshold(p, tau, k0)
+        S, _ = select_threshold(p, tau, k0, gs)
     else:
         raise ValueError(f"unknown mode {mode}")
     ids, w = refine(p, S, k)

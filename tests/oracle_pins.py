@@ -20,7 +20,10 @@ the oracle disagrees with what the paper or the mathematics fixes:
   the smallest superset of S_0 covering a fraction tau of the score mass;
 * the layer stack of Eq. 1: the budget split, bf16 rounding against torch and
   hand-derived double-rounding cases, the residual identity, budget = N per
-  layer as a plain top-k stack.
+  layer as a plain top-k stack;
+* the sparse-score reading of Sec. 2.2: the gating rows are the plain top-k
+  routing weights, a hand-derived example, S inside the union of the top-k
+  sets, greedy optimality by brute force, and budget = N as plain top-k.
 
 `test_oracle_pins.py` runs them on the oracle; `test_oracle_mutations.py`
 plants mistakes in the oracle and checks that some pin fails.
@@ -610,6 +613,80 @@ def check_stack_invariants(O):
     assert not np.array_equal(a[-1], x)
 
 
+# ---------------------------------------------------------------- Sec. 2.2: sparse gating scores
+
+def check_topk_gating(O):
+    """Sec. 2.2's g has k nonzeros per token, proportional to p on the token's
+    top-k and summing to 1; they equal plain top-k routing's weights; and a
+    hand-derived example."""
+    rng = np.random.default_rng(8)
+    p = W_softmax(rng, 20, 40)
+    for k in (1, 3, 8):
+        g = O.topk_gating(p, k)
+        r = O.route(p, k, 0, O.MODE_TOPK)
+        assert np.all((g > 0).sum(axis=1) == k)
+        for i in range(p.shape[0]):
+            nz = sorted(np.nonzero(g[i])[0].tolist())
+            assert nz == sorted(lexsort_top(p[i], k, range(p.shape[1])))
+            assert np.array_equal(g[i, r["ids"][i]], r["w"][i])     # same fp32 values
+            assert abs(float(np.sum(g[i].astype(np.float64))) - 1.0) < 1e-6
+    # p = [0.5, 0.25, 0.125, 0.125], k = 2: T = {0, 1}, D = 0.75,
+    # g = [fp32(0.5/0.75), fp32(0.25/0.75), 0, 0] = [0x3f2aaaab, 0x3eaaaaab, 0, 0]
+    g = O.topk_gating(np.array([[0.5, 0.25, 0.125, 0.125]], dtype=np.float32), 2)
+    assert [hex(int(v)) for v in g[0].view(np.uint32)] == ["0x3f2aaaab", "0x3eaaaaab", "0x0", "0x0"]
+
+
+def W_softmax(rng, B, N, scale=1.5):
+    h = rng.standard_normal((B, N)) * scale
+    return (np.exp(h) / np.exp(h).sum(axis=1, keepdims=True)).astype(np.float32)
+
+
+def check_sparse_selection(O, cases=30):
+    """With sparse scores: S is S_0 plus only experts some token ranks in its
+    top-k; |S| = |S_0| + min(m, available); among supersets of S_0 of that
+    size S maximises the sparse objective (brute force); budget N gives plain
+    top-k routing exactly."""
+    rng = np.random.default_rng(17)
+    done = 0
+    while done < cases:
+        N = int(rng.integers(4, 10))
+        B = int(rng.integers(1, 6))
+        k = int(rng.integers(1, min(N, 4) + 1))
+        k0 = int(rng.integers(0, k + 1))
+        m = int(rng.integers(0, N + 1))
+        p = quantised_scores(rng, B, N)
+        g = O.topk_gating(p, k)
+        union = set()
+        for i in range(B):
+            union |= set(lexsort_top(p[i], k, range(N)))
+        S0 = set()
+        for i in range(B):
+            S0 |= set(lexsort_top(p[i], k0, range(N)))
+        S = mask_to_set(O.route(p, k, m, O.MODE_BATCH, k0=k0, sparse_scores=1)["mask"])
+        assert S0 <= S <= (S0 | union)
+        avail = [j for j in union if j not in S0]
+        assert len(S) == len(S0) + min(m, len(avail))
+        col = exact_colsum(g, range(B))
+        best = max(sum((col[j] for j in c), Fraction(0))
+                   for c in itertools.combinations(avail, len(S) - len(S0)))
+        assert sum((col[j] for j in S - S0), Fraction(0)) == best
+        done += 1
+    for trial in range(5):
+        B, N, k = 12, 24, 4
+        p = W_softmax(rng, B, N)
+        a = O.route(p, k, N, O.MODE_BATCH, k0=1, sparse_scores=1)
+        b = O.route(p, k, 0, O.MODE_TOPK)
+        assert np.array_equal(a["ids"], b["ids"]) and np.array_equal(a["w"], b["w"])
+        assert a["n_selected"] == b["union_topk"]
+        for mode, prm in ((O.MODE_GROUP, dict(n_groups=4, m_g=N)),
+                          (O.MODE_HIER, dict(m_r=N, tokens_per_request=3))):
+            c = O.route(p, k, N, mode, k0=1, sparse_scores=1, **prm)
+            assert mask_to_set(c["mask"]) == mask_to_set(a["mask"]), mode
+        # tau = 1 stops once the running fp32 sum reaches f(E): never beyond the union
+        c = O.route(p, k, 0, O.MODE_THRESH, k0=1, sparse_scores=1, tau=1.0)
+        assert mask_to_set(c["mask"]) <= mask_to_set(a["mask"])
+
+
 ALL_CHECKS = [
     check_closed_form_golden, check_union_statistics, check_greedy_bruteforce,
     check_hier_bruteforce, check_hier_single_request_is_batch, check_group,
@@ -618,4 +695,5 @@ ALL_CHECKS = [
     check_combine_multi_token, check_canonical_sum_golden, check_canonical_sum_bound,
     check_threshold_golden, check_threshold_bruteforce, check_threshold_consistency,
     check_bf16_rounding, check_layer_budgets, check_stack_invariants,
+    check_topk_gating, check_sparse_selection,
 ]

@@ -199,6 +199,19 @@ def _bf16_via_fp32(x):
     return _orig["f64_to_bf16_bits"](x.astype(np.float64))
 
 
+def _gating_unnormalised(p, k):
+    p = np.asarray(p, dtype=np.float32)
+    g = np.zeros_like(p)
+    for i in range(p.shape[0]):
+        for j in O.top(p[i], k, range(p.shape[1])):
+            g[i, j] = p[i, j]
+    return g
+
+
+def _candidates_allow_zero(scores, S, positive_only, pool=None):
+    return _orig["candidates"](scores, S, False, pool)
+
+
 def _closed_form_wrong(N, k, B):
     return N * (1.0 - (1.0 - k / N) ** (B - 1))
 
@@ -232,6 +245,8 @@ MUTATIONS = {
     "budget split drops the remainder": ("layer_budgets", _budgets_floor),
     "bf16 by truncation": ("f64_to_bf16_bits", _bf16_truncate),
     "bf16 rounded through fp32": ("f64_to_bf16_bits", _bf16_via_fp32),
+    "sparse gating not renormalised": ("topk_gating", _gating_unnormalised),
+    "sparse selection adds zero-gain experts": ("candidates", _candidates_allow_zero),
 }
 
 _orig = {name: getattr(O, name) for name, _ in MUTATIONS.values()}
