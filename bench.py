@@ -64,6 +64,8 @@ def parse_args(argv=None):
     ap.add_argument("--k0", type=int, default=None)
     ap.add_argument("--mode", default=None, choices=sorted(W.MODES))
     ap.add_argument("--tau", type=float, default=None, help="covered score-mass fraction (thresh)")
+    ap.add_argument("--sparse", action="store_true",
+                    help="column scores from the top-k-masked gating values (Sec. 2.2)")
     ap.add_argument("--shared", type=int, default=0,
                     help="shared experts added to every token (DeepSeek-R1 has one)")
     ap.add_argument("--layers", type=int, default=1,
@@ -94,6 +96,8 @@ def workload_from_args(args) -> W.Workload:
         kw["mode"] = W.MODES[args.mode]
     if args.tau is not None:
         kw["tau"] = args.tau
+    if args.sparse:
+        kw["sparse_scores"] = 1
     return w.with_(**kw) if kw else w
 
 
@@ -109,6 +113,8 @@ def describe(w: W.Workload, n_shared: int = 0) -> str:
         s += f" G={w.n_groups} m_g={w.m_g} k0={w.k0}"
     elif w.mode == W.MODE_THRESH:
         s += f" tau={w.tau} k0={w.k0}"
+    if w.sparse_scores:
+        s += ", sparse (top-k-masked) column scores"
     if n_shared:
         s += f" + {n_shared} shared expert{'s' if n_shared > 1 else ''}"
     return s
@@ -623,7 +629,8 @@ def cpu_baseline(w: W.Workload, seed: int, n_shared: int = 0) -> dict:
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
                CUDA_VISIBLE_DEVICES="")
     f_rows = max(128, w.F // 4)
-    kw = json.dumps(dict(B=w.B, N=w.N, F=w.F, budget=w.budget, k0=w.k0, mode=w.mode, tau=w.tau))
+    kw = json.dumps(dict(B=w.B, N=w.N, F=w.F, budget=w.budget, k0=w.k0, mode=w.mode, tau=w.tau,
+                         sparse_scores=w.sparse_scores))
     code = (f"import sys, json; sys.path.insert(0, {ROOT!r}); import torch; torch.set_num_threads(1); "
             f"import bench; from paper_2602_07265_gb300 import workloads as W; "
             f"w = W.WORKLOADS[{w.name!r}].with_(**{kw}); "

@@ -85,6 +85,13 @@ typedef struct {
                                  max_group_load statistic in every mode; 0 = 1 */
   int32_t m_g;                /* GROUP: per-group budget m_g (Algorithm 5) */
   float tau;                  /* THRESH: covered fraction of the score mass, 0 <= tau <= 1 */
+  int32_t sparse_scores;      /* 0: column scores sum the dense softmax g (default).
+                                 1: they sum Sec. 2.2's top-k-masked gating values
+                                 g_ij = p_ij / D_i on the token's Top k (D_i = fp32 sum
+                                 of those k scores in rank order, 1/k each if D_i = 0),
+                                 0 elsewhere, and an expert whose column score is 0 is
+                                 never added (no gain).  Warm-up and refinement use the
+                                 dense scores in both.  Ignored by TOPK. */
 } xs_route_params;
 
 /* Per-call statistics, written by the device into caller memory. */
@@ -101,7 +108,7 @@ typedef struct {
 /* Host-side error codes (return values). */
 #define XS_OK 0
 #define XS_ERR_SHAPE (-1)     /* B, N, k, d or F out of range or misaligned */
-#define XS_ERR_PARAM (-2)     /* mode, budget, k0, m_r, m_g, n_groups, tokens_per_request or tau invalid */
+#define XS_ERR_PARAM (-2)     /* mode, budget or a field of xs_route_params invalid */
 #define XS_ERR_NULL (-3)      /* a required pointer is NULL */
 #define XS_ERR_WORKSPACE (-4) /* workspace NULL, too small or not 256-byte aligned */
 #define XS_ERR_ALIGN (-5)     /* a tensor pointer is not 16-byte aligned */
@@ -191,6 +198,7 @@ int xshare_moe_forward(const uint16_t *x, const float *W_g, const uint16_t *W_ga
  * on every GPU that loads the library, held until the process exits), so:
  *   - B is limited to 1024 tokens (N <= 1024 and k <= 16 as elsewhere); a
  *     larger B returns XS_ERR_SHAPE and launches nothing;
+ *   - only the dense scores: prm->sparse_scores != 0 returns XS_ERR_PARAM;
  *   - the first call on a device looks up the array's device address with
  *     cudaGetSymbolAddress; make that first call before any stream capture;
  *   - every call on a device uses the same array, so calls that can overlap

@@ -44,6 +44,7 @@ int check_route_args(int B, int N, int k, int budget, int mode, const xs_route_p
   if (B < 1 || B > kMaxB || N < 1 || N > kMaxN || k < 1 || k > kMaxK || k > N) return XS_ERR_SHAPE;
   if (mode < XS_MODE_TOPK || mode > XS_MODE_THRESH) return XS_ERR_PARAM;
   if (mode == XS_MODE_THRESH && !(prm->tau >= 0.f && prm->tau <= 1.f)) return XS_ERR_PARAM;
+  if (prm->sparse_scores != 0 && prm->sparse_scores != 1) return XS_ERR_PARAM;
   if (budget < 0 || prm->k0 < 0 || prm->k0 > kMaxK || prm->k0 > N || prm->m_r < 0 || prm->m_g < 0 ||
       prm->n_groups < 0)
     return XS_ERR_PARAM;
@@ -83,6 +84,8 @@ RouteArgs route_args(const Plan &pl, void *ws, int B, int N, int k, int budget, 
   a.G = prm->n_groups < 1 ? 1 : prm->n_groups;
   a.m_g = prm->m_g > N ? N : prm->m_g;
   a.tau = prm->tau;
+  a.sparse = (mode != XS_MODE_TOPK) ? prm->sparse_scores : 0;
+  a.gs = at<float>(ws, pl.gs);
   a.p = at<float>(ws, pl.p);
   a.mask = at<uint8_t>(ws, pl.mask);
   a.ids = at<int32_t>(ws, pl.ids);
@@ -131,6 +134,7 @@ Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms, int 
   pl.chunk_col = take((size_t)chunks * N * 4);
   pl.chunk_marks = take((size_t)chunks * 2 * N);
   pl.done = take(4 * sizeof(int32_t));
+  pl.gs = take((size_t)B * N * 4);
   if (with_ffn) {
     pl.xp = take((size_t)pl.max_rows * d * 2);
     pl.act = take((size_t)pl.max_rows * F * 2);

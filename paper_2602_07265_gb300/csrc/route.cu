@@ -490,7 +490,9 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
                   [](int, int) { return true; });
     lane_sort<kQ>(L);
     int32_t *top = a.toptok + (size_t)t * kMaxK;
-    lane_take<kQ>(L, kk, [&](int r, int id, float) {
+    int my_id = -1;  // sparse scores: lane s keeps slot s of the token's top-k
+    float my_v = 0.f, D = 0.f;
+    lane_take<kQ>(L, kk, [&](int r, int id, float v) {
       if (lane == 0) {
         if (r < k) s_union[id] = 1;
         if (r < a.k0) {
@@ -501,7 +503,30 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
             s_base[id] = 1;
         }
       }
+      if (r < k) {
+        if (lane == r) {
+          my_id = id;
+          my_v = v;
+        }
+        D = __fadd_rn(D, v);  // rank order, identical on every lane
+      }
     });
+    if (a.sparse) {
+      // Sec. 2.2's gating values replace the dense row for the column sums:
+      // p / D on the token's top-k, 0 elsewhere (1/k each if D = 0).
+      float *grow = (hier && !hier_here) ? a.gs + (size_t)t * N : nullptr;
+      __syncwarp();
+      for (int j = lane; j < N; j += 32) {
+        prow_s[j] = 0.f;
+        if (grow) grow[j] = 0.f;
+      }
+      __syncwarp();
+      if (lane < k) {
+        const float gv = (D > 0.f) ? __fdiv_rn(my_v, D) : __fdiv_rn(1.f, (float)k);
+        prow_s[my_id] = gv;
+        if (grow) grow[my_id] = gv;
+      }
+    }
   }
   __syncthreads();
 
@@ -543,7 +568,9 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
         }
       LaneList<kQ> L;
       lane_load<kQ>(L, 0, N, lane, [&](int q, int) { return sc[q]; },
-                    [&](int q, int) { return ((excl >> q) & 1u) == 0; });
+                    [&](int q, int) {
+                      return ((excl >> q) & 1u) == 0 && (!a.sparse || sc[q] > 0.f);
+                    });
       lane_sort<kQ>(L);
       lane_take<kQ>(L, a.m_r, [&](int, int id, float) {
         if (lane == 0) s_base[id] = 1;
@@ -592,7 +619,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
 #pragma unroll
       for (int q = 0; q < kQ; ++q) {
         const int j = lane + 32 * q;
-        sc[q] = (j < N) ? canonical_sum(a.p, N, j, r0, r1) : 0.f;
+        sc[q] = (j < N) ? canonical_sum(a.sparse ? a.gs : a.p, N, j, r0, r1) : 0.f;
       }
       for (int x = r0; x < r1; ++x)
         for (int i = 0; i < a.k0; ++i) {
@@ -604,7 +631,9 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
         }
       LaneList<kQ> L;
       lane_load<kQ>(L, 0, N, lane, [&](int q, int) { return sc[q]; },
-                    [&](int q, int) { return ((excl >> q) & 1u) == 0; });
+                    [&](int q, int) {
+                      return ((excl >> q) & 1u) == 0 && (!a.sparse || sc[q] > 0.f);
+                    });
       lane_sort<kQ>(L);
       lane_take<kQ>(L, a.m_r, [&](int, int id, float) {
         if (lane == 0) s_base[id] = 1;
@@ -626,7 +655,8 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
     const int n_base = __syncthreads_count(tid < N && s_base[tid]);
     for (int g = warp; g < G; g += nwarps) {
       int cnt = 0;
-      for (int j = g * size + lane; j < (g + 1) * size; j += 32) cnt += s_base[j] ? 0 : 1;
+      for (int j = g * size + lane; j < (g + 1) * size; j += 32)
+        cnt += (s_base[j] == 0 && (!a.sparse || s_col[j] > 0.f)) ? 1 : 0;
       cnt = __reduce_add_sync(kFull, cnt);
       if (lane == 0) s_gl[g] = cnt;
     }
@@ -650,7 +680,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
       for (int g = warp; g < G; g += nwarps) {
         LaneList<kQ> L;
         lane_load<kQ>(L, g * size, size, lane, [&](int, int j) { return s_col[j]; },
-                      [&](int, int j) { return s_base[j] == 0; });
+                      [&](int, int j) { return s_base[j] == 0 && (!a.sparse || s_col[j] > 0.f); });
         lane_sort<kQ>(L);
         lane_take<kQ>(L, R, [&](int, int id, float) {
           if (lane == 0) s_mask[id] = 1;
@@ -672,7 +702,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
       float f = expert_tree<kQ>(v0);
       LaneList<kQ> L;
       lane_load<kQ>(L, 0, N, lane, [&](int, int j) { return s_col[j]; },
-                    [&](int, int j) { return s_base[j] == 0; });
+                    [&](int, int j) { return s_base[j] == 0 && (!a.sparse || s_col[j] > 0.f); });
       lane_sort<kQ>(L);
       while (f < target) {
         float v = 0.f;
@@ -691,7 +721,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
     // `budget` best experts outside the base set by the batch column score.
     LaneList<kQ> L;
     lane_load<kQ>(L, 0, N, lane, [&](int, int j) { return s_col[j]; },
-                  [&](int, int j) { return s_base[j] == 0; });
+                  [&](int, int j) { return s_base[j] == 0 && (!a.sparse || s_col[j] > 0.f); });
     lane_sort<kQ>(L);
     lane_take<kQ>(L, a.budget, [&](int, int id, float) {
       if (lane == 0) s_mask[id] = 1;
@@ -725,7 +755,8 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   refine_tokens<kQ>(
       a, s_mask, 0, B, min(k, nsel),
       [&](int t) -> const float * {
-        return (t >= t0 && t < t0 + nt) ? ps + (t - t0) * N : a.p + (size_t)t * N;
+        // The chunk's rows hold the sparse values in that mode; refine on dense p.
+        return (t >= t0 && t < t0 + nt && !a.sparse) ? ps + (t - t0) * N : a.p + (size_t)t * N;
       },
       ids_s);
   if (C > 1) __threadfence();

@@ -62,6 +62,7 @@ extern "C" int xshare_route_static(const float *scores, int B, int N, int k, int
     return XS_ERR_SHAPE;
   if (mode < XS_MODE_TOPK || mode > XS_MODE_THRESH) return XS_ERR_PARAM;
   if (mode == XS_MODE_THRESH && !(prm->tau >= 0.f && prm->tau <= 1.f)) return XS_ERR_PARAM;
+  if (prm->sparse_scores != 0) return XS_ERR_PARAM;  // the dense reading only
   if (budget < 0 || prm->k0 < 0 || prm->k0 > kMaxK || prm->k0 > N || prm->m_r < 0 ||
       prm->m_g < 0 || prm->n_groups < 0)
     return XS_ERR_PARAM;

@@ -77,7 +77,7 @@ struct Meta {
 // Byte offsets of every workspace region (256-byte aligned).
 struct Plan {
   size_t h, p, mask, ids, w, toptok, counts, offsets, perm, pos, tiles, meta;
-  size_t chunk_col, chunk_marks, done;
+  size_t chunk_col, chunk_marks, done, gs;
   size_t xp, act, out, ffn_part, ffn_cnt;
   size_t total;
   int max_pairs;   // routed pairs B * k
@@ -92,6 +92,8 @@ struct RouteArgs {
   float *p;              // [B, N] scores (input if logits == nullptr, else output)
   int B, N, k, budget, mode, k0, m_r, T, G, m_g;
   float tau;             // THRESH: covered fraction of the score mass
+  int sparse;            // column scores from the top-k-masked gating values
+  float *gs;             // [B, N] those values, written when HIER needs them from global
   uint8_t *mask;         // [N]
   int32_t *ids;          // [B, k]
   float *w;              // [B, k]

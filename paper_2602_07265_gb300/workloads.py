@@ -56,6 +56,7 @@ class Workload:
     n_groups: int = 1   # G (GROUP)
     m_g: int = 0        # per-group budget (GROUP)
     tau: float = 0.0    # covered score-mass fraction (THRESH)
+    sparse_scores: int = 0  # column scores from the top-k-masked gating values
     x_kind: str = "iid"  # "iid" | "request" | "domains"
     n_domains: int = 4
     domain_std: float = 1.5
@@ -64,7 +65,8 @@ class Workload:
 
     def params(self) -> Dict[str, int]:
         return dict(k0=self.k0, m_r=self.m_r, tokens_per_request=self.tokens_per_request,
-                    n_groups=self.n_groups, m_g=self.m_g, tau=self.tau)
+                    n_groups=self.n_groups, m_g=self.m_g, tau=self.tau,
+                    sparse_scores=self.sparse_scores)
 
     def with_(self, **kw) -> "Workload":
         return dataclasses.replace(self, **kw)

@@ -35,7 +35,8 @@ class RouteParams(ctypes.Structure):
     """xs_route_params."""
     _fields_ = [("k0", ctypes.c_int32), ("m_r", ctypes.c_int32),
                 ("tokens_per_request", ctypes.c_int32), ("n_groups", ctypes.c_int32),
-                ("m_g", ctypes.c_int32), ("tau", ctypes.c_float)]
+                ("m_g", ctypes.c_int32), ("tau", ctypes.c_float),
+                ("sparse_scores", ctypes.c_int32)]
 
 
 class SharedExperts(ctypes.Structure):
@@ -55,8 +56,8 @@ class Layer(ctypes.Structure):
 
 
 def route_params(k0: int = 0, m_r: int = 0, tokens_per_request: int = 1, n_groups: int = 1,
-                 m_g: int = 0, tau: float = 0.0) -> RouteParams:
-    return RouteParams(k0, m_r, tokens_per_request, n_groups, m_g, tau)
+                 m_g: int = 0, tau: float = 0.0, sparse_scores: int = 0) -> RouteParams:
+    return RouteParams(k0, m_r, tokens_per_request, n_groups, m_g, tau, sparse_scores)
 
 
 def _load() -> ctypes.CDLL:

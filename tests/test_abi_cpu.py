@@ -84,7 +84,7 @@ def test_route_rejects_bad_arguments(X, kw, code):
     (dict(tokens_per_request=0), 3, -2), (dict(tokens_per_request=3), 3, -2),
     (dict(tokens_per_request=16), 3, -2),
     (dict(tau=-0.1), 4, -2), (dict(tau=1.5), 4, -2), (dict(tau=float("nan")), 4, -2),
-    (dict(), 5, -2),
+    (dict(), 5, -2), (dict(sparse_scores=2), 1, -2), (dict(sparse_scores=-1), 1, -2),
 ])
 def test_route_rejects_bad_params(X, prm, mode, code):
     assert _route_rc(X, mode=mode, prm=X.route_params(**prm)) == code
@@ -141,3 +141,10 @@ def test_stack_rejects_bad_arguments(X):
     assert not out.value
     assert X.LIB.xshare_stack_graph_launch(None, None) == -3
     X.LIB.xshare_stack_graph_destroy(None)
+
+
+def test_route_static_rejects_sparse_scores(X):
+    P = 1 << 20
+    prm = X.route_params(sparse_scores=1)
+    assert X.LIB.xshare_route_static(P, 8, 16, 4, 4, 1, ctypes.byref(prm), P, P, P, None, None,
+                                     None, None, None) == -2

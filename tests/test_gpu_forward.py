@@ -162,6 +162,7 @@ SMALL = [
     W.QWEN3, W.QWEN3.with_(B=16, m_r=5), W.QWEN3.with_(k0=0, budget=16),
     W.QWEN3.with_(mode=W.MODE_TOPK),
     W.TINY.with_(mode=W.MODE_THRESH, tau=0.5, k0=1), W.OLMOE.with_(mode=W.MODE_THRESH, tau=0.7),
+    W.OLMOE.with_(B=32, budget=24, sparse_scores=1), W.QWEN3.with_(sparse_scores=1),
 ]
 
 
@@ -178,7 +179,8 @@ def test_forward_parity_small(X, case, seed):
 @pytest.mark.parametrize("w", [
     W.DSR1.with_(B=8), W.DSR1, W.DSR1.with_(B=128, budget=64), W.DSR1.with_(k0=0, budget=32),
     W.DSR1_GROUP, W.DSR1_GROUP.with_(k0=0, m_g=8), W.DSR1.with_(mode=W.MODE_THRESH, tau=0.5),
-], ids=lambda w: f"{w.name}-B{w.B}-m{w.budget}-k0{w.k0}-mg{w.m_g}-mode{w.mode}")
+    W.DSR1.with_(budget=40, sparse_scores=1),
+], ids=lambda w: f"{w.name}-B{w.B}-m{w.budget}-k0{w.k0}-mg{w.m_g}-mode{w.mode}-s{w.sparse_scores}")
 def test_forward_parity_full_size_sampled(X, w):
     """DeepSeek-R1-shaped layers at full size; the oracle checks sampled tokens."""
     x, W_g = W.router_inputs(w, 0)

@@ -30,8 +30,8 @@ def X():
 def gpu_route(X, p: np.ndarray, k: int, budget: int, mode: int, **params):
     B, N = p.shape
     dev = torch.device("cuda")
-    prm = X.route_params(**{**dict(k0=0, m_r=0, tokens_per_request=1, n_groups=1, m_g=0, tau=0.0),
-                            **params})
+    prm = X.route_params(**{**dict(k0=0, m_r=0, tokens_per_request=1, n_groups=1, m_g=0, tau=0.0,
+                                   sparse_scores=0), **params})
     ws = torch.empty(X.xshare_workspace_size(B, N, k, 0, 0, mode, prm), dtype=torch.uint8, device=dev)
     scores = torch.from_numpy(np.ascontiguousarray(p)).to(dev)
     out = dict(
@@ -75,7 +75,7 @@ def oracle_scores(w: W.Workload, seed: int) -> np.ndarray:
 
 
 def check(X, p, k, budget, mode, **params):
-    full = dict(k0=0, m_r=0, tokens_per_request=1, n_groups=1, m_g=0, tau=0.0)
+    full = dict(k0=0, m_r=0, tokens_per_request=1, n_groups=1, m_g=0, tau=0.0, sparse_scores=0)
     full.update(params)
     ref = O.route(p, k, budget, mode, **full)
     g = gpu_route(X, p, k, budget, mode, **full)
@@ -227,3 +227,36 @@ def test_threshold_zero_scores(X):
     check(X, p, 8, 0, W.MODE_THRESH, k0=0, tau=1.0)
     p[:] = 0.0
     check(X, p, 8, 0, W.MODE_THRESH, k0=0, tau=0.5)
+
+
+# ---- sparse-score reading (Sec. 2.2's top-k-masked g in the column sums) ----
+@pytest.mark.parametrize("case", range(len(WL_CASES)))
+def test_sparse_scores_route_parity(X, case):
+    w, _ = WL_CASES[case]
+    p = oracle_scores(w, 5)
+    ref = check(X, p, w.k, w.budget, w.mode, **{**w.params(), "sparse_scores": 1})
+    assert ref["n_selected"] <= ref["union_topk"] + len(O.warmup_set(p, w.k0, range(w.B)))
+
+
+@pytest.mark.parametrize("B,N,k,budget,mode,params", [
+    (32, 64, 8, 64, W.MODE_BATCH, dict(k0=1)),                         # budget beyond the union
+    (33, 1000, 16, 100, W.MODE_BATCH, dict(k0=16)),
+    (96, 128, 8, 2, W.MODE_HIER, dict(k0=1, m_r=3, tokens_per_request=3)),   # straddling requests
+    (144, 64, 4, 5, W.MODE_HIER, dict(k0=2, m_r=2, tokens_per_request=48)),
+    (256, 256, 8, 0, W.MODE_GROUP, dict(k0=1, n_groups=8, m_g=40)),     # groups run out of gain
+    (64, 256, 8, 0, W.MODE_THRESH, dict(k0=1, tau=0.9)),
+    (2048, 256, 8, 32, W.MODE_BATCH, dict(k0=1)),
+    (40, 50, 8, 20, W.MODE_BATCH, dict(k0=0)),
+])
+def test_sparse_scores_edge_cases(X, B, N, k, budget, mode, params):
+    for ties in (False, True):
+        p = W.random_scores(B, N, seed=B + 3 * N, ties=ties)
+        check(X, p, k, budget, mode, sparse_scores=1, **params)
+
+
+def test_sparse_budget_n_is_plain_topk(X):
+    p = W.random_scores(64, 128, seed=4)
+    a = gpu_route(X, p, 8, 128, W.MODE_BATCH, k0=1, sparse_scores=1)
+    b = gpu_route(X, p, 8, 0, W.MODE_TOPK)
+    assert np.array_equal(a["ids"], b["ids"]) and np.array_equal(a["w"], b["w"])
+    assert a["stats"]["n_selected"] == b["stats"]["union_topk"]
