@@ -136,6 +136,7 @@ Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms, int 
   pl.done = take(4 * sizeof(int32_t));
   pl.gs = take((size_t)B * N * 4);
   if (with_ffn) {
+    pl.rstat = take((size_t)router_tc_ctas(B, N, d, n_sms) * 4);
     pl.xp = take((size_t)pl.max_rows * d * 2);
     pl.act = take((size_t)pl.max_rows * F * 2);
     pl.out = take((size_t)pl.max_rows * d * 4);
@@ -269,8 +270,17 @@ int xs::forward_impl(const FwdCall &c, FwdStep step) {
            cudaEventRecord(reinterpret_cast<cudaEvent_t>(events[i]), s) == cudaSuccess;
   };
   if (!mark(0)) return XS_ERR_CUDA;
-  if (launch_router_logits(c.x, c.W_g, h, B, N, d, a.done, s) != cudaSuccess || !mark(1))
-    return XS_ERR_CUDA;
+  cudaError_t re;
+  if (B >= kRouterTcMinB) {
+    int32_t *rstat = at<int32_t>(workspace, pl.rstat);
+    int grid = 0;
+    re = launch_router_tc(c.x, c.W_g, h, B, N, d, a.done, rstat, sms, &grid, s);
+    a.router_status = rstat;
+    a.router_ctas = grid;
+  } else {
+    re = launch_router_logits(c.x, c.W_g, h, B, N, d, a.done, s);
+  }
+  if (re != cudaSuccess || !mark(1)) return XS_ERR_CUDA;
   a.events = events ? events + 2 : nullptr;  // between the selection and refinement kernels
   if (launch_route(a, s) != cudaSuccess || !mark(3)) return XS_ERR_CUDA;
   if (launch_gather(c.x, a.perm, a.meta, const_cast<uint16_t *>(f.xp), pl.max_rows, B, d, k,

@@ -397,7 +397,7 @@ __device__ void build_permutation(const RouteArgs &a, PermSmem sm) {
       st.union_topk = m.union_topk;
       st.max_group_load = m.max_group_load;
       st.n_pairs = m.n_pairs;
-      st.status = 0;
+      st.status = m.status;
       st.reserved[0] = st.reserved[1] = 0;
       *a.stats = st;
     }
@@ -733,6 +733,9 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   if (tid == 0) s_gl[kMaxN] = 0;
   selection_stats(a, s_mask, s_union, s_gl, nsel, n_union, maxload);
   for (int j = tid; j < N; j += blockDim.x) a.mask[j] = s_mask[j];
+  int rstat = 0;  // the router's status, if it reports one
+  for (int i = tid; i < a.router_ctas; i += blockDim.x) rstat = max(rstat, __ldcg(a.router_status + i));
+  rstat = __syncthreads_or(rstat);
   if (tid == 0) {
     Meta m;
     for (int i = 0; i < 7; ++i) m.pad[i] = 0;
@@ -744,7 +747,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
     m.n_used = 0;
     m.union_topk = n_union;
     m.max_group_load = maxload;
-    m.status = 0;
+    m.status = rstat ? XS_DEV_TIMEOUT : XS_DEV_OK;
     *a.meta = m;
   }
   if (!a.fuse_refine) return;

@@ -77,7 +77,7 @@ struct Meta {
 // Byte offsets of every workspace region (256-byte aligned).
 struct Plan {
   size_t h, p, mask, ids, w, toptok, counts, offsets, perm, pos, tiles, meta;
-  size_t chunk_col, chunk_marks, done, gs;
+  size_t chunk_col, chunk_marks, done, gs, rstat;
   size_t xp, act, out, ffn_part, ffn_cnt;
   size_t total;
   int max_pairs;   // routed pairs B * k
@@ -116,11 +116,20 @@ struct RouteArgs {
   void *const *events;   // nullable: events[0] is recorded between the two kernels
   int fuse_refine;       // set by launch_route: refinement runs in the selection kernel
   int n_shared;          // shared-expert tiles appended after the routed ones
+  const int32_t *router_status;  // nullable: per-CTA status of the tensor-core router
+  int router_ctas;
 };
 
 cudaError_t launch_route(const RouteArgs &a, cudaStream_t s);
 cudaError_t launch_router_logits(const uint16_t *x, const float *Wg, float *h, int B, int N,
                                  int d, int32_t *done, cudaStream_t s);
+// The router on the tensor cores (router_tc.cu).  status: [router_tc_ctas()]
+// words, an upper bound on its grid; each launched CTA writes its word.
+constexpr int kRouterTcMinB = 64;   // batches from this size use it
+int router_tc_ctas(int B, int N, int d, int n_sms);
+cudaError_t launch_router_tc(const uint16_t *x, const float *Wg, float *h, int B, int N, int d,
+                             int32_t *done, int32_t *status, int n_sms, int *grid_out,
+                             cudaStream_t s);
 cudaError_t launch_combine(const float *out, const int32_t *pos, const float *w,
                            const Meta *meta, const uint16_t *resid, uint16_t *y, int B, int d,
                            int k, int n_shared, cudaStream_t s);

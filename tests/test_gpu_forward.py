@@ -270,3 +270,24 @@ def test_forward_shared_experts_full_size_sampled(X):
     g0 = gpu_forward(X, w, x, W_g, weights)
     assert np.array_equal(g0["ids"], g["ids"]) and np.array_equal(g0["p"], g["p"])
     assert not np.array_equal(g0["y"], g["y"])
+
+
+# ---- router logits on either path (CUDA cores below 64 tokens, tensor cores from 64) ----
+@pytest.mark.parametrize("w", [
+    W.TINY.with_(B=63), W.TINY.with_(B=64), W.TINY.with_(B=65, budget=16),
+    W.OLMOE.with_(B=200), W.QWEN3.with_(B=1000, tokens_per_request=8),
+    W.DSR1.with_(B=256, budget=40),
+], ids=lambda w: f"{w.name}-B{w.B}")
+def test_router_scores_both_paths(X, w):
+    """The dense scores from the router and softmax are within P_RTOL of the
+    oracle's (fp64 logits, fp32 softmax), elementwise, and repeat bit for bit."""
+    x, W_g = W.router_inputs(w, 2)
+    weights = device_weights(w, 2)
+    a = gpu_forward(X, w, x, W_g, weights)
+    b = gpu_forward(X, w, x, W_g, weights)
+    assert np.array_equal(a["p"], b["p"]) and np.array_equal(a["y"], b["y"])
+    assert a["stats"]["status"] == 0
+    ref = O.softmax_scores(O.router_logits(W.bf16_bits(x), W_g.numpy()))
+    rel = np.abs(a["p"].astype(np.float64) - ref) / ref.astype(np.float64)
+    print(f"[{w.name} B={w.B}] router+softmax max rel {rel.max():.2e}")
+    assert rel.max() <= P_RTOL
