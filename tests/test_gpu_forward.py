@@ -291,3 +291,17 @@ def test_router_scores_both_paths(X, w):
     rel = np.abs(a["p"].astype(np.float64) - ref) / ref.astype(np.float64)
     print(f"[{w.name} B={w.B}] router+softmax max rel {rel.max():.2e}")
     assert rel.max() <= P_RTOL
+
+
+# ---- limits: the largest batch and expert count, the smallest d and F ----
+@pytest.mark.parametrize("w,tokens", [
+    (W.TINY.with_(B=8192, budget=24, k0=1), [0, 4095, 8191]),           # B at the limit
+    (W.TINY.with_(N=1024, k=16, budget=64, k0=2, B=96), None),           # N and k at the limit
+    (W.TINY.with_(d=128, F=128, B=80, budget=8), None),                  # smallest d and F
+    (W.TINY.with_(N=1000, k=8, budget=40, B=130, n_groups=8), None),    # N not a multiple of 32
+])
+def test_forward_limits(X, w, tokens):
+    x, W_g = W.router_inputs(w, 7)
+    weights = device_weights(w, 7)
+    g = gpu_forward(X, w, x, W_g, weights)
+    compare(w, g, x, W_g, weights, tokens=tokens)
