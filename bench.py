@@ -74,6 +74,8 @@ def parse_args(argv=None):
                     help="distinct expert-weight sets the stack's layers cycle through")
     ap.add_argument("--global-budget", type=int, default=None,
                     help="stack budget K (default: layers x the per-layer budget)")
+    ap.add_argument("--unpacked", action="store_true",
+                    help="read the expert weights as plain [N, F, d] matrices instead of packed tiles")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--seed", type=int, default=0)
     return ap.parse_args(argv)
@@ -240,15 +242,21 @@ class ClockSampler:
 
 # --------------------------------------------------------------------------- traffic
 
-def kernel_source_hash() -> str:
-    """Hash of the kernel sources: a recorded ncu traffic figure is only valid
-    for the sources it was captured from."""
+# The source files each timed stage's kernel is built from.
+KERNEL_SOURCES = {
+    "ffn_gate_up": ("ffn_tc.cu", "tc_ptx.cuh", "tmap.cu", "tmap.cuh", "xs_internal.cuh"),
+    "ffn_down": ("ffn_tc.cu", "tc_ptx.cuh", "tmap.cu", "tmap.cuh", "xs_internal.cuh"),
+}
+
+
+def kernel_source_hash(stage: str = "ffn_gate_up") -> str:
+    """Hash of the sources of one stage's kernel: a recorded ncu traffic figure
+    is only valid for the sources it was captured from."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2602_07265_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh")):
-            with open(os.path.join(csrc, name), "rb") as f:
-                h.update(name.encode() + f.read())
+    for name in KERNEL_SOURCES[stage]:
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + f.read())
     return h.hexdigest()[:16]
 
 
@@ -261,7 +269,7 @@ def recorded_traffic(stage: str, units: float):
             rec = json.load(f).get(stage)
     except (OSError, ValueError):
         return None
-    if not rec or rec.get("source_hash") != kernel_source_hash():
+    if not rec or stage not in KERNEL_SOURCES or rec.get("source_hash") != kernel_source_hash(stage):
         return None
     return float(rec["bytes_per_unit"]) * units
 
@@ -301,6 +309,12 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
     Wg, Wu, Wd = W.expert_weights(w, args.seed, device=str(dev))
     Ns = args.shared
     shared = W.shared_expert_weights(w, Ns, args.seed, device=str(dev)) if Ns else None
+    packed = not args.unpacked
+    if packed:  # a layout change made once when the weights are loaded, outside the timed region
+        pk = X.Packed(Wg, Wu, Wd)
+        pshared = X.Packed(*shared) if shared is not None else None
+        del Wg, Wu, Wd
+        torch.cuda.empty_cache()
     prm = X.route_params(**w.params())
     ws = torch.empty(X.xshare_workspace_size(w.B, w.N, w.k, w.d, w.F, w.mode, prm, Ns),
                      dtype=torch.uint8, device=dev)
@@ -309,9 +323,16 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
     stats = torch.zeros(K, X.STATS_WORDS, dtype=torch.int32, device=dev)
     events = [[torch.cuda.Event(enable_timing=True) for _ in range(X.N_STAGES + 1)] for _ in range(K)]
 
+    def forward(x_in, st=None, ev=None):
+        if packed:
+            X.xshare_moe_forward_packed(x_in, W_g, pk, w.k, w.budget, w.mode, prm, y, ws,
+                                        shared=pshared, stats=st, stage_events=ev)
+        else:
+            X.xshare_moe_forward(x_in, W_g, Wg, Wu, Wd, w.k, w.budget, w.mode, prm, y, ws,
+                                 stats=st, stage_events=ev, shared=shared)
+
     def step(i, st=None, ev=None):
-        X.xshare_moe_forward(xs_dev[i % N_ROTATE], W_g, Wg, Wu, Wd, w.k, w.budget, w.mode, prm,
-                             y, ws, stats=st, stage_events=ev, shared=shared)
+        forward(xs_dev[i % N_ROTATE], st, ev)
 
     for i in range(Wm):
         step(i)
@@ -371,8 +392,7 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
 
     def e2e_step(i):
         x_in.copy_(x_pin[i % N_ROTATE], non_blocking=True)
-        X.xshare_moe_forward(x_in, W_g, Wg, Wu, Wd, w.k, w.budget, w.mode, prm, y, ws, stats=st_dev,
-                             shared=shared)
+        forward(x_in, st_dev)
         y_pin.copy_(y, non_blocking=True)
         st_pin.copy_(st_dev, non_blocking=True)
         stream.synchronize()
@@ -409,6 +429,8 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
         "config": {
             "workload": describe(w, Ns),
             "B": w.B, "N": w.N, "k": w.k, "d": w.d, "F": w.F, "shared_experts": Ns,
+            "expert_weights": "packed 128 x 64 tiles (xshare_pack_experts, once at load)"
+                              if packed else "plain [N, F, d] / [N, d, F] matrices",
             "global_batch": w.B * world,
             "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
             "l2": f"inputs larger than L2: ~{layer_bytes / 1e9:.2f} GB of expert weights per step "
@@ -467,10 +489,17 @@ def run_gpu_stack(args, w: W.Workload, rank: int, world: int, local: int) -> dic
     shared = [W.shared_expert_weights(w, Ns, args.seed + 10 * s, device=str(dev),
                                       down_std=W.STACK_DOWN_STD) if Ns else None
               for s in range(P)]
+    if not args.unpacked:  # packed once at load, outside the timed region
+        sets = [X.Packed(*ws) for ws in sets]
+        shared = [X.Packed(*sh) if sh is not None else None for sh in shared]
+        torch.cuda.empty_cache()
     layers = []
     for l in range(L):
         _, W_g = W.router_inputs(w, args.seed + 1000 + l)
-        layers.append((W_g.to(dev),) + tuple(sets[l % P]) + (shared[l % P],))
+        if args.unpacked:
+            layers.append((W_g.to(dev),) + tuple(sets[l % P]) + (shared[l % P],))
+        else:
+            layers.append((W_g.to(dev), sets[l % P], shared[l % P]))
     x_host = W.router_inputs(w, args.seed + 101 * rank)[0]
     x = x_host.to(dev)
     prm = X.route_params(**w.params())
@@ -546,6 +575,7 @@ def run_gpu_stack(args, w: W.Workload, rank: int, world: int, local: int) -> dic
                         f"global budget K={K_total} (m_l = K/L), {P} expert-weight sets, "
                         "one CUDA-graph replay per step",
             "B": w.B, "N": w.N, "k": w.k, "d": w.d, "F": w.F, "layers": L, "weight_sets": P,
+            "expert_weights": "plain matrices" if args.unpacked else "packed tiles",
             "global_budget": K_total, "shared_experts": Ns, "global_batch": w.B * world,
             "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
             "l2": f"inputs larger than L2: ~{stack_bytes / 1e9:.1f} GB of expert weights per step",

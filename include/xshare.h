@@ -130,6 +130,20 @@ typedef struct {
   int32_t n_shared;           /* 0 .. 8 */
 } xs_shared_experts;
 
+/* Expert weights packed for the FFN's weight stream (xshare_pack_experts):
+ * every 128-row x 64-column tile the tensor cores consume, stored contiguously
+ * in the order the kernels read it and already in the shared-memory layout
+ * (128-byte swizzle), so a pipeline stage's weights arrive in one contiguous
+ * bulk copy.  Same bytes as the unpacked matrices:
+ *   gate_up: n * F * d * 2 bf16 (gate and up tiles interleaved),
+ *   down   : n * d * F bf16.
+ * Device pointers, 16-byte aligned. */
+typedef struct {
+  const void *gate_up;
+  const void *down;
+  int32_t n;                  /* experts (for shared experts: 0 .. 8) */
+} xs_packed_experts;
+
 /* Bytes of workspace the calls below need for these sizes.  For
  * xshare_route pass d = F = 0 and n_shared = 0.  Returns 0 for arguments the
  * calls would reject.  Depends on the current device's SM count. */
@@ -233,18 +247,41 @@ int xshare_moe_forward_profiled(const uint16_t *x, const float *W_g, const uint1
                                 void *workspace, size_t ws_bytes, xs_stream_t stream,
                                 void *const *stage_events);
 
+/* Packs n experts' weights (W_gate, W_up [n, F, d], W_down [n, d, F] bf16,
+ * device) into the layout of xs_packed_experts: gate_up (n F d 2 bf16) and
+ * down (n d F bf16), caller-allocated device buffers that must not overlap
+ * the inputs.  d, F multiples of 128.  A layout change only, done once per
+ * set of weights (no counterpart in the paper).  Asynchronous on `stream`. */
+int xshare_pack_experts(const uint16_t *W_gate, const uint16_t *W_up, const uint16_t *W_down, int n,
+                        int d, int F, void *gate_up, void *down, xs_stream_t stream);
+
+/* xshare_moe_forward on packed expert weights: `experts` holds the N routed
+ * experts (experts->n == N), `shared` (nullable) the shared ones.  Results
+ * are identical, bit for bit, to xshare_moe_forward on the unpacked weights.
+ * stage_events: NULL, or XS_N_STAGES + 1 events as in
+ * xshare_moe_forward_profiled. */
+int xshare_moe_forward_packed(const uint16_t *x, const float *W_g, const xs_packed_experts *experts,
+                              int B, int d, int F, int N, int k, int budget, int mode,
+                              const xs_route_params *prm, const xs_packed_experts *shared,
+                              uint16_t *y, float *scores_out, uint8_t *sel_mask, int32_t *topk_ids,
+                              float *topk_w, xs_stats *stats, void *workspace, size_t ws_bytes,
+                              xs_stream_t stream, void *const *stage_events);
+
 /* Name of stage i of xshare_moe_forward (e.g. "router"), or "" if out of range. */
 const char *xshare_stage_name(int i);
 
 /* One MoE layer of a stack: router W_g [N, d] fp32, experts as in
- * xshare_moe_forward, optional shared experts (NULL: none).  Device pointers;
- * several layers may point to the same weights. */
+ * xshare_moe_forward, optional shared experts (NULL: none), or the packed
+ * forms of both.  Device pointers; several layers may point to the same
+ * weights. */
 typedef struct {
   const float *W_g;
   const uint16_t *W_gate;
   const uint16_t *W_up;
   const uint16_t *W_down;
   const xs_shared_experts *shared;
+  const xs_packed_experts *packed;         /* nullable: packed experts, used instead of W_* */
+  const xs_packed_experts *packed_shared;  /* nullable: packed shared experts (with `packed`) */
 } xs_layer;
 
 /* A stack of L MoE layers under one global expert budget (Eq. 1 at the system

@@ -203,18 +203,28 @@ int xs::forward_impl(const FwdCall &c, FwdStep step) {
   if (rc != XS_OK) return rc;
   rc = check_ffn_shape(d, F);
   if (rc != XS_OK) return rc;
-  if (!c.x || !c.W_g || !c.W_gate || !c.W_up || !c.W_down || !c.y) return XS_ERR_NULL;
-  if (!aligned16(c.x) || !aligned16(c.W_g) || !aligned16(c.W_gate) || !aligned16(c.W_up) ||
-      !aligned16(c.W_down) || !aligned16(c.y) || (c.scores_out && !aligned16(c.scores_out)) ||
-      (c.resid && !aligned16(c.resid)))
+  const bool packed = c.P_gate_up != nullptr || c.P_down != nullptr;
+  if (!c.x || !c.W_g || !c.y) return XS_ERR_NULL;
+  if (packed ? (!c.P_gate_up || !c.P_down) : (!c.W_gate || !c.W_up || !c.W_down)) return XS_ERR_NULL;
+  if (!aligned16(c.x) || !aligned16(c.W_g) || !aligned16(c.y) ||
+      (c.scores_out && !aligned16(c.scores_out)) || (c.resid && !aligned16(c.resid)))
+    return XS_ERR_ALIGN;
+  if (packed ? (!aligned16(c.P_gate_up) || !aligned16(c.P_down))
+             : (!aligned16(c.W_gate) || !aligned16(c.W_up) || !aligned16(c.W_down)))
     return XS_ERR_ALIGN;
   const xs_shared_experts *shared = c.shared;
-  const int n_shared = shared ? shared->n_shared : 0;
+  const xs_packed_experts *pshared = c.packed_shared;
+  if (packed && shared && shared->n_shared != 0) return XS_ERR_PARAM;  // packed calls take packed ones
+  const int n_shared = packed ? (pshared ? pshared->n : 0) : (shared ? shared->n_shared : 0);
   if (n_shared < 0 || n_shared > kMaxShared) return XS_ERR_PARAM;
-  if (n_shared > 0) {
+  if (n_shared > 0 && !packed) {
     if (!shared->W_gate || !shared->W_up || !shared->W_down) return XS_ERR_NULL;
     if (!aligned16(shared->W_gate) || !aligned16(shared->W_up) || !aligned16(shared->W_down))
       return XS_ERR_ALIGN;
+  }
+  if (n_shared > 0 && packed) {
+    if (!pshared->gate_up || !pshared->down) return XS_ERR_NULL;
+    if (!aligned16(pshared->gate_up) || !aligned16(pshared->down)) return XS_ERR_ALIGN;
   }
   void *workspace = c.workspace;
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return XS_ERR_WORKSPACE;
@@ -244,7 +254,12 @@ int xs::forward_impl(const FwdCall &c, FwdStep step) {
   f.W_gate = c.W_gate;
   f.W_up = c.W_up;
   f.W_down = c.W_down;
-  if (n_shared > 0) {
+  f.P_gate_up = c.P_gate_up;
+  f.P_down = c.P_down;
+  if (n_shared > 0 && packed) {
+    f.PS_gate_up = pshared->gate_up;
+    f.PS_down = pshared->down;
+  } else if (n_shared > 0) {
     f.S_gate = shared->W_gate;
     f.S_up = shared->W_up;
     f.S_down = shared->W_down;
@@ -365,6 +380,47 @@ extern "C" int xshare_moe_forward_profiled(const uint16_t *x, const float *W_g,
                                 shared, y, scores_out, sel_mask, topk_ids, topk_w, stats,
                                 workspace, ws_bytes, stream, stage_events),
                       FwdStep::kLaunch);
+}
+
+extern "C" int xshare_moe_forward_packed(const uint16_t *x, const float *W_g,
+                                         const xs_packed_experts *experts, int B, int d, int F,
+                                         int N, int k, int budget, int mode,
+                                         const xs_route_params *prm,
+                                         const xs_packed_experts *shared, uint16_t *y,
+                                         float *scores_out, uint8_t *sel_mask, int32_t *topk_ids,
+                                         float *topk_w, xs_stats *stats, void *workspace,
+                                         size_t ws_bytes, xs_stream_t stream,
+                                         void *const *stage_events) {
+  if (experts == nullptr || experts->gate_up == nullptr || experts->down == nullptr) return XS_ERR_NULL;
+  if (experts->n != N) return XS_ERR_SHAPE;
+  if (stage_events != nullptr)
+    for (int i = 0; i <= XS_N_STAGES; ++i)
+      if (stage_events[i] == nullptr) return XS_ERR_NULL;
+  FwdCall c = make_call(x, W_g, nullptr, nullptr, nullptr, B, d, F, N, k, budget, mode, prm, nullptr,
+                        y, scores_out, sel_mask, topk_ids, topk_w, stats, workspace, ws_bytes, stream,
+                        stage_events);
+  c.P_gate_up = experts->gate_up;
+  c.P_down = experts->down;
+  c.packed_shared = shared;
+  return forward_impl(c, FwdStep::kLaunch);
+}
+
+extern "C" int xshare_pack_experts(const uint16_t *W_gate, const uint16_t *W_up, const uint16_t *W_down,
+                                   int n, int d, int F, void *gate_up, void *down, xs_stream_t stream) {
+  if (n < 1 || n > kMaxN) return XS_ERR_SHAPE;
+  int rc = check_ffn_shape(d, F);
+  if (rc != XS_OK) return rc;
+  if (!W_gate || !W_up || !W_down || !gate_up || !down) return XS_ERR_NULL;
+  if (!aligned16(W_gate) || !aligned16(W_up) || !aligned16(W_down) || !aligned16(gate_up) ||
+      !aligned16(down))
+    return XS_ERR_ALIGN;
+  const int sms = current_device_sms();
+  if (sms < 0) return sms;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (launch_pack(W_gate, W_up, gate_up, n, F, d, sms, s) != cudaSuccess ||
+      launch_pack(W_down, nullptr, down, n, d, F, sms, s) != cudaSuccess)
+    return XS_ERR_CUDA;
+  return XS_OK;
 }
 
 extern "C" const char *xshare_stage_name(int i) {

@@ -66,6 +66,8 @@ struct TcParams {
   CUtensorMap tmS1;
   CUtensorMap tmB[4];   // xp (gate/up) or act (down): [max_rows, K] bf16, boxes of
                         // 16, 32, 64, 128 rows x 64
+  const uint8_t *pk;        // nullable: packed weights (pack.cu); then tmA0 / tmA1 are unused
+  const uint8_t *pk_shared; // packed shared experts
   const Tile *tiles;
   Meta *meta;
   xs_stats *stats;
@@ -147,11 +149,13 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
     fence_mbar_init();
-    prefetch_tmap(&p.tmA0);
-    if (kGateUp) prefetch_tmap(&p.tmA1);
-    if (p.has_shared) {
-      prefetch_tmap(&p.tmS0);
-      if (kGateUp) prefetch_tmap(&p.tmS1);
+    if (p.pk == nullptr) {
+      prefetch_tmap(&p.tmA0);
+      if (kGateUp) prefetch_tmap(&p.tmA1);
+      if (p.has_shared) {
+        prefetch_tmap(&p.tmS0);
+        if (kGateUp) prefetch_tmap(&p.tmS1);
+      }
     }
     for (int i = 0; i < 4; ++i) prefetch_tmap(&p.tmB[i]);
   }
@@ -184,7 +188,13 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
         const bool routed = tl.expert < p.n_routed;
         const CUtensorMap *mA0 = routed ? &p.tmA0 : &p.tmS0;
         const CUtensorMap *mA1 = routed ? &p.tmA1 : &p.tmS1;
-        const int arow = (routed ? tl.expert : tl.expert - p.n_routed) * p.M + mt * kBM;
+        const int e_local = routed ? tl.expert : tl.expert - p.n_routed;
+        const int arow = e_local * p.M + mt * kBM;
+        // Packed weights: the unit's blocks are consecutive, one per K step.
+        const uint8_t *pblk =
+            p.pk ? (routed ? p.pk : p.pk_shared) +
+                       ((static_cast<size_t>(e_local) * MT + mt) * KI) * (C::kNumA * kTileBytes)
+                 : nullptr;
         for (int kk = k0; kk < k1; ++kk) {
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, kWaitNs, abort_flag)) {
             ok = false;
@@ -193,8 +203,13 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
           const uint32_t sA = sbase + stage * C::kStageBytes;
           const uint32_t sB = sA + C::kNumA * kTileBytes;
           mbar_arrive_expect_tx(full_bar(stage), tx);
-          tma_load_2d(sA, mA0, full_bar(stage), kk * kBK, arow, pol_w);
-          if (kGateUp) tma_load_2d(sA + kTileBytes, mA1, full_bar(stage), kk * kBK, arow, pol_w);
+          if (pblk) {
+            bulk_load(sA, pblk + static_cast<size_t>(kk) * (C::kNumA * kTileBytes), C::kNumA * kTileBytes,
+                      full_bar(stage), pol_w);
+          } else {
+            tma_load_2d(sA, mA0, full_bar(stage), kk * kBK, arow, pol_w);
+            if (kGateUp) tma_load_2d(sA + kTileBytes, mA1, full_bar(stage), kk * kBK, arow, pol_w);
+          }
           tma_load_2d(sB, &p.tmB[bsel], full_bar(stage), kk * kBK, tl.row0, pol_x);
           issued_mask |= 1u << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
@@ -422,15 +437,19 @@ size_t ffn_cnt_words(int max_tiles, int B, int d, int F) {
 cudaError_t launch_ffn_gate_up(const FfnArgs &a, cudaStream_t s) {
   TcParams p;
   memset(&p, 0, sizeof(p));
-  if (!make_map(&p.tmA0, a.W_gate, a.d, static_cast<uint64_t>(a.N) * a.F, kBM) ||
-      !make_map(&p.tmA1, a.W_up, a.d, static_cast<uint64_t>(a.N) * a.F, kBM) ||
-      !make_token_maps(p.tmB, a.xp, a.d, a.max_rows))
+  if (!make_token_maps(p.tmB, a.xp, a.d, a.max_rows)) return cudaErrorInvalidValue;
+  if (a.P_gate_up != nullptr) {
+    p.pk = static_cast<const uint8_t *>(a.P_gate_up);
+    p.pk_shared = static_cast<const uint8_t *>(a.PS_gate_up);
+  } else if (!make_map(&p.tmA0, a.W_gate, a.d, static_cast<uint64_t>(a.N) * a.F, kBM) ||
+             !make_map(&p.tmA1, a.W_up, a.d, static_cast<uint64_t>(a.N) * a.F, kBM)) {
     return cudaErrorInvalidValue;
-  if (a.n_shared > 0) {
+  }
+  if (a.n_shared > 0 && a.P_gate_up == nullptr) {
     if (!make_map(&p.tmS0, a.S_gate, a.d, static_cast<uint64_t>(a.n_shared) * a.F, kBM) ||
         !make_map(&p.tmS1, a.S_up, a.d, static_cast<uint64_t>(a.n_shared) * a.F, kBM))
       return cudaErrorInvalidValue;
-  } else {
+  } else if (a.P_gate_up == nullptr) {
     p.tmS0 = p.tmA0;
     p.tmS1 = p.tmA1;
   }
@@ -451,15 +470,20 @@ cudaError_t launch_ffn_gate_up(const FfnArgs &a, cudaStream_t s) {
 cudaError_t launch_ffn_down(const FfnArgs &a, cudaStream_t s) {
   TcParams p;
   memset(&p, 0, sizeof(p));
-  if (!make_map(&p.tmA0, a.W_down, a.F, static_cast<uint64_t>(a.N) * a.d, kBM) ||
-      !make_token_maps(p.tmB, a.act, a.F, a.max_rows))
-    return cudaErrorInvalidValue;
-  p.tmA1 = p.tmA0;
-  if (a.n_shared > 0) {
-    if (!make_map(&p.tmS0, a.S_down, a.F, static_cast<uint64_t>(a.n_shared) * a.d, kBM))
-      return cudaErrorInvalidValue;
+  if (!make_token_maps(p.tmB, a.act, a.F, a.max_rows)) return cudaErrorInvalidValue;
+  if (a.P_down != nullptr) {
+    p.pk = static_cast<const uint8_t *>(a.P_down);
+    p.pk_shared = static_cast<const uint8_t *>(a.PS_down);
   } else {
-    p.tmS0 = p.tmA0;
+    if (!make_map(&p.tmA0, a.W_down, a.F, static_cast<uint64_t>(a.N) * a.d, kBM))
+      return cudaErrorInvalidValue;
+    p.tmA1 = p.tmA0;
+    if (a.n_shared > 0) {
+      if (!make_map(&p.tmS0, a.S_down, a.F, static_cast<uint64_t>(a.n_shared) * a.d, kBM))
+        return cudaErrorInvalidValue;
+    } else {
+      p.tmS0 = p.tmA0;
+    }
   }
   p.tmS1 = p.tmS0;
   p.n_routed = a.N;

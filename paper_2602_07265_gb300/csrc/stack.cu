@@ -43,6 +43,13 @@ FwdCall layer_call(const uint16_t *x, const xs_layer *layers, int L, int l, int 
   c.W_up = layers[l].W_up;
   c.W_down = layers[l].W_down;
   c.shared = layers[l].shared;
+  if (layers[l].packed != nullptr) {
+    c.W_gate = c.W_up = c.W_down = nullptr;
+    c.P_gate_up = layers[l].packed->gate_up;
+    c.P_down = layers[l].packed->down;
+    c.packed_shared = layers[l].packed_shared;
+    c.shared = nullptr;
+  }
   c.B = B;
   c.d = d;
   c.F = F;
@@ -75,6 +82,8 @@ int stack_run(const uint16_t *x, const xs_layer *layers, int L, int B, int d, in
     const size_t act = static_cast<size_t>(B) * d * 2;
     if (overlaps(x, act, h_out, act * L)) return XS_ERR_PARAM;
   }
+  for (int l = 0; l < L; ++l)
+    if (layers[l].packed != nullptr && layers[l].packed->n != N) return XS_ERR_SHAPE;
   for (FwdStep step : {FwdStep::kCheckArgs, FwdStep::kCheckAll, FwdStep::kLaunch}) {
     if (step == FwdStep::kLaunch && !launch) break;
     for (int l = 0; l < L; ++l) {

@@ -139,6 +139,8 @@ cudaError_t launch_gather(const uint16_t *x, const int32_t *perm, const Meta *me
 struct FfnArgs {
   const uint16_t *W_gate, *W_up, *W_down;
   const uint16_t *S_gate, *S_up, *S_down;   // shared experts, used when n_shared > 0
+  // Packed weights (pack.cu), nullable; when set they replace the matrices above.
+  const void *P_gate_up, *P_down, *PS_gate_up, *PS_down;
   int n_shared;
   const uint16_t *xp;    // [max_rows, d] permuted token rows
   uint16_t *act;         // [max_rows, F] silu(g) * u, bf16
@@ -154,6 +156,9 @@ struct FfnArgs {
 cudaError_t launch_ffn_gate_up(const FfnArgs &a, cudaStream_t s);
 cudaError_t launch_ffn_down(const FfnArgs &a, cudaStream_t s);
 size_t ffn_part_bytes(int n_sms);
+// Packs W0 (and W1) [n][M][K] bf16 into 128 x 64 swizzled tiles (pack.cu).
+cudaError_t launch_pack(const uint16_t *W0, const uint16_t *W1, void *P, int n, int M, int K,
+                        int n_sms, cudaStream_t s);
 size_t ffn_cnt_words(int max_tiles, int B, int d, int F);
 
 // One MoE-layer forward as the C entry points describe it, plus `resid`
@@ -166,6 +171,8 @@ struct FwdCall {
   const xs_route_params *prm;
   const xs_shared_experts *shared;
   const uint16_t *resid;
+  const void *P_gate_up, *P_down;          // nullable: packed weights instead of W_gate/W_up/W_down
+  const xs_packed_experts *packed_shared;  // nullable: packed shared experts
   uint16_t *y;
   float *scores_out;
   uint8_t *sel_mask;

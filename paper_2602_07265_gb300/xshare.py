@@ -48,11 +48,18 @@ class SharedExperts(ctypes.Structure):
 MAX_SHARED = 8
 
 
+class PackedExperts(ctypes.Structure):
+    """xs_packed_experts (device pointers and count)."""
+    _fields_ = [("gate_up", ctypes.c_void_p), ("down", ctypes.c_void_p), ("n", ctypes.c_int32)]
+
+
 class Layer(ctypes.Structure):
-    """xs_layer (device pointers; `shared` points to an SharedExperts or is NULL)."""
+    """xs_layer (device pointers; `shared`, `packed`, `packed_shared` may be NULL)."""
     _fields_ = [("W_g", ctypes.c_void_p), ("W_gate", ctypes.c_void_p),
                 ("W_up", ctypes.c_void_p), ("W_down", ctypes.c_void_p),
-                ("shared", ctypes.POINTER(SharedExperts))]
+                ("shared", ctypes.POINTER(SharedExperts)),
+                ("packed", ctypes.POINTER(PackedExperts)),
+                ("packed_shared", ctypes.POINTER(PackedExperts))]
 
 
 def route_params(k0: int = 0, m_r: int = 0, tokens_per_request: int = 1, n_groups: int = 1,
@@ -80,6 +87,12 @@ def _load() -> ctypes.CDLL:
     lib.xshare_route_static.restype = I
     lib.xshare_moe_forward_profiled.argtypes = lib.xshare_moe_forward.argtypes + [P]
     lib.xshare_moe_forward_profiled.restype = I
+    PP = ctypes.POINTER(PackedExperts)
+    lib.xshare_pack_experts.argtypes = [P, P, P, I, I, I, P, P, P]
+    lib.xshare_pack_experts.restype = I
+    lib.xshare_moe_forward_packed.argtypes = [P, P, PP, I, I, I, I, I, I, I, PR, PP,
+                                              P, P, P, P, P, P, P, Z, P, P]
+    lib.xshare_moe_forward_packed.restype = I
     PL = ctypes.POINTER(Layer)
     lib.xshare_stack_forward.argtypes = [P, PL, I, I, I, I, I, I, I, I, PR, P, P, P, Z, P]
     lib.xshare_stack_forward.restype = I
@@ -237,22 +250,92 @@ def xshare_moe_forward(x: torch.Tensor, W_g: torch.Tensor, W_gate: torch.Tensor,
     _check(LIB.xshare_moe_forward_profiled(*args, handles), "xshare_moe_forward_profiled")
 
 
+class Packed:
+    """Packed expert weights (xshare_pack_experts) on the device: gate_up and
+    down byte buffers plus the expert count, d and F."""
+
+    def __init__(self, W_gate: torch.Tensor, W_up: torch.Tensor, W_down: torch.Tensor, stream=None):
+        n, F, d = W_gate.shape
+        if tuple(W_up.shape) != (n, F, d) or tuple(W_down.shape) != (n, d, F):
+            raise ValueError("W_gate, W_up [n, F, d] and W_down [n, d, F]")
+        self.n, self.d, self.F = n, d, F
+        self.gate_up = torch.empty(n * F * d * 2 * 2, dtype=torch.uint8, device=W_gate.device)
+        self.down = torch.empty(n * d * F * 2, dtype=torch.uint8, device=W_gate.device)
+        _check(LIB.xshare_pack_experts(_ptr(W_gate, torch.bfloat16, "W_gate"),
+                                       _ptr(W_up, torch.bfloat16, "W_up"),
+                                       _ptr(W_down, torch.bfloat16, "W_down"), n, d, F,
+                                       self.gate_up.data_ptr(), self.down.data_ptr(),
+                                       _stream(stream)), "xshare_pack_experts")
+
+    def struct(self) -> PackedExperts:
+        return PackedExperts(self.gate_up.data_ptr(), self.down.data_ptr(), self.n)
+
+
+def xshare_moe_forward_packed(x: torch.Tensor, W_g: torch.Tensor, experts: Packed, k: int,
+                              budget: int, mode: int, params: RouteParams, y: torch.Tensor,
+                              workspace: torch.Tensor, shared: Optional[Packed] = None,
+                              scores_out: Optional[torch.Tensor] = None,
+                              sel_mask: Optional[torch.Tensor] = None,
+                              topk_ids: Optional[torch.Tensor] = None,
+                              topk_w: Optional[torch.Tensor] = None,
+                              stats: Optional[torch.Tensor] = None, stream=None,
+                              stage_events: Optional[list] = None) -> None:
+    """xshare_moe_forward on packed expert weights; see xshare.h."""
+    B, d = x.shape
+    N = W_g.shape[0]
+    if experts.n != N or experts.d != d or tuple(y.shape) != (B, d) or W_g.shape[1] != d:
+        raise ValueError("inconsistent shapes")
+    ex = experts.struct()
+    sh = shared.struct() if shared is not None else None
+    handles = None
+    if stage_events is not None:
+        if len(stage_events) != N_STAGES + 1:
+            raise ValueError(f"stage_events needs {N_STAGES + 1} events")
+        handles = (ctypes.c_void_p * (N_STAGES + 1))()
+        for i, ev in enumerate(stage_events):
+            if not ev.cuda_event:
+                ev.record()
+            handles[i] = ev.cuda_event
+    rc = LIB.xshare_moe_forward_packed(
+        _ptr(x, torch.bfloat16, "x"), _ptr(W_g, torch.float32, "W_g"), ctypes.byref(ex), B, d,
+        experts.F, N, k, budget, mode, ctypes.byref(params),
+        ctypes.byref(sh) if sh is not None else None, _ptr(y, torch.bfloat16, "y"),
+        _ptr(scores_out, torch.float32, "scores_out", B * N),
+        _ptr(sel_mask, torch.uint8, "sel_mask", N), _ptr(topk_ids, torch.int32, "topk_ids", B * k),
+        _ptr(topk_w, torch.float32, "topk_w", B * k), _ptr(stats, torch.int32, "stats", STATS_WORDS),
+        _ptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream), handles)
+    _check(rc, "xshare_moe_forward_packed")
+
+
 def _stack_args(x, layers, k, K_total, mode, params, h_out, workspace, stats):
     """Marshals a layer stack: `layers` is a list of (W_g, W_gate, W_up, W_down)
-    or (W_g, W_gate, W_up, W_down, (S_gate, S_up, S_down)) tensors."""
+    or (W_g, W_gate, W_up, W_down, (S_gate, S_up, S_down)) tensors, or of
+    (W_g, Packed[, Packed shared]) for packed expert weights."""
     B, d = x.shape
     L = len(layers)
     if L < 1:
         raise ValueError("at least one layer")
-    N, F = layers[0][1].shape[0], layers[0][1].shape[1]
+    first = layers[0][1]
+    N, F = (first.n, first.F) if isinstance(first, Packed) else (first.shape[0], first.shape[1])
     arr = (Layer * L)()
     keep = []
     for l, lay in enumerate(layers):
-        W_g, Wg, Wu, Wd = lay[:4]
-        if W_g.shape != (N, d) or tuple(Wg.shape) != (N, F, d) or tuple(Wu.shape) != (N, F, d) \
-                or tuple(Wd.shape) != (N, d, F):
-            raise ValueError(f"layer {l}: inconsistent shapes")
+        W_g = lay[0]
+        if W_g.shape != (N, d):
+            raise ValueError(f"layer {l}: W_g must be [N, d]")
         arr[l].W_g = _ptr(W_g, torch.float32, "W_g")
+        if isinstance(lay[1], Packed):
+            pk = lay[1].struct()
+            keep.append(pk)
+            arr[l].packed = ctypes.pointer(pk)
+            if len(lay) > 2 and lay[2] is not None:
+                ps = lay[2].struct()
+                keep.append(ps)
+                arr[l].packed_shared = ctypes.pointer(ps)
+            continue
+        Wg, Wu, Wd = lay[1:4]
+        if tuple(Wg.shape) != (N, F, d) or tuple(Wu.shape) != (N, F, d) or tuple(Wd.shape) != (N, d, F):
+            raise ValueError(f"layer {l}: inconsistent shapes")
         arr[l].W_gate = _ptr(Wg, torch.bfloat16, "W_gate")
         arr[l].W_up = _ptr(Wu, torch.bfloat16, "W_up")
         arr[l].W_down = _ptr(Wd, torch.bfloat16, "W_down")

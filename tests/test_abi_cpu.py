@@ -27,7 +27,8 @@ def declared_functions():
 
 
 def test_header_declares_the_boundary():
-    assert declared_functions() == ["xshare_moe_forward", "xshare_moe_forward_profiled",
+    assert declared_functions() == ["xshare_moe_forward", "xshare_moe_forward_packed",
+                                    "xshare_moe_forward_profiled", "xshare_pack_experts",
                                     "xshare_route", "xshare_route_static",
                                     "xshare_selftest_wait_timeout", "xshare_stack_forward",
                                     "xshare_stack_graph_create", "xshare_stack_graph_destroy",
@@ -148,3 +149,24 @@ def test_route_static_rejects_sparse_scores(X):
     prm = X.route_params(sparse_scores=1)
     assert X.LIB.xshare_route_static(P, 8, 16, 4, 4, 1, ctypes.byref(prm), P, P, P, None, None,
                                      None, None, None) == -2
+
+
+def test_packed_entry_points_reject_bad_arguments(X):
+    P = 1 << 20
+    assert X.LIB.xshare_pack_experts(P, P, P, 0, 256, 256, P, P, None) == -1
+    assert X.LIB.xshare_pack_experts(P, P, P, 4, 100, 256, P, P, None) == -1
+    assert X.LIB.xshare_pack_experts(P, None, P, 4, 256, 256, P, P, None) == -3
+    assert X.LIB.xshare_pack_experts(P, P, P, 4, 256, 256, P + 8, P, None) == -5
+    prm = X.route_params()
+    ex = X.PackedExperts(P, P, 16)
+    def rc(ex=ex, sh=None, ev=None):
+        return X.LIB.xshare_moe_forward_packed(P, P, ctypes.byref(ex) if ex is not None else None,
+                                               4, 256, 256, 16, 2, 2, 1, ctypes.byref(prm),
+                                               ctypes.byref(sh) if sh is not None else None,
+                                               P, None, None, None, None, None, P, 1 << 20, None, ev)
+    assert rc(ex=None) == -3
+    assert rc(ex=X.PackedExperts(P, P, 15)) == -1          # count must equal N
+    assert rc(ex=X.PackedExperts(P, None, 16)) == -3
+    assert rc(ex=X.PackedExperts(P + 4, P, 16)) == -5
+    assert rc(sh=X.PackedExperts(P, P, 9)) == -2
+    assert rc(sh=X.PackedExperts(None, P, 1)) == -3
