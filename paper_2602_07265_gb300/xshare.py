@@ -17,7 +17,7 @@ import torch
 
 from . import _build
 
-MODE_TOPK, MODE_BATCH, MODE_GROUP, MODE_HIER = 0, 1, 2, 3
+MODE_TOPK, MODE_BATCH, MODE_GROUP, MODE_HIER, MODE_THRESH = 0, 1, 2, 3, 4
 MODES = {"topk": MODE_TOPK, "batch": MODE_BATCH, "group": MODE_GROUP, "hier": MODE_HIER}
 
 XS_DEV_OK, XS_DEV_TIMEOUT = 0, 1
