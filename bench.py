@@ -64,6 +64,8 @@ def parse_args(argv=None):
     ap.add_argument("--k0", type=int, default=None)
     ap.add_argument("--mode", default=None, choices=sorted(W.MODES))
     ap.add_argument("--tau", type=float, default=None, help="covered score-mass fraction (thresh)")
+    ap.add_argument("--m-r", type=int, default=None, help="per-request budget (hier)")
+    ap.add_argument("--m-g", type=int, default=None, help="per-group budget (group)")
     ap.add_argument("--sparse", action="store_true",
                     help="column scores from the top-k-masked gating values (Sec. 2.2)")
     ap.add_argument("--shared", type=int, default=0,
@@ -98,6 +100,10 @@ def workload_from_args(args) -> W.Workload:
         kw["mode"] = W.MODES[args.mode]
     if args.tau is not None:
         kw["tau"] = args.tau
+    if args.m_r is not None:
+        kw["m_r"] = args.m_r
+    if args.m_g is not None:
+        kw["m_g"] = args.m_g
     if args.sparse:
         kw["sparse_scores"] = 1
     return w.with_(**kw) if kw else w
@@ -660,7 +666,7 @@ def cpu_baseline(w: W.Workload, seed: int, n_shared: int = 0) -> dict:
                CUDA_VISIBLE_DEVICES="")
     f_rows = max(128, w.F // 4)
     kw = json.dumps(dict(B=w.B, N=w.N, F=w.F, budget=w.budget, k0=w.k0, mode=w.mode, tau=w.tau,
-                         sparse_scores=w.sparse_scores))
+                         sparse_scores=w.sparse_scores, m_r=w.m_r, m_g=w.m_g))
     code = (f"import sys, json; sys.path.insert(0, {ROOT!r}); import torch; torch.set_num_threads(1); "
             f"import bench; from paper_2602_07265_gb300 import workloads as W; "
             f"w = W.WORKLOADS[{w.name!r}].with_(**{kw}); "
