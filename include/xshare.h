@@ -10,9 +10,12 @@
  *   - Device pointers point to memory of the current CUDA device, row-major and
  *     contiguous, at least 16-byte aligned unless stated otherwise.  bf16
  *     tensors are passed as uint16_t (the raw bf16 bit pattern).
- *   - The caller owns every buffer.  The library allocates nothing: scratch
+ *   - The caller owns every buffer.  The library does not allocate: scratch
  *     space is the caller's `workspace` of at least xshare_workspace_size()
- *     bytes, 256-byte aligned, which the calls overwrite.
+ *     bytes, 256-byte aligned, which the calls overwrite.  Two exceptions,
+ *     stated at their declarations: xshare_route_static uses a fixed array
+ *     inside the library, and xshare_stack_graph_create lets CUDA allocate
+ *     the graph it instantiates.
  *   - Calls are asynchronous and stream-ordered on `stream` (a cudaStream_t;
  *     NULL is the legacy default stream).  No call synchronises the stream or
  *     the device.  Two calls that share a workspace must not overlap.
@@ -24,7 +27,14 @@
  *   - Scores must be finite (no NaN): selection compares them as fp32 values.
  *
  * Limits: 1 <= N <= 1024 experts; 1 <= k <= min(N, 16); 0 <= k0 <= min(N, 16);
- * 1 <= B <= 8192 tokens; for xshare_moe_forward d % 128 == 0 and F % 128 == 0.
+ * 1 <= B <= 8192 tokens; for the forward calls d % 128 == 0 and F % 128 == 0;
+ * at most 8 shared experts.
+ *
+ * Entry points: xshare_route (selection and refinement on given scores) and
+ * its workspace-free variant; xshare_moe_forward (the whole layer), on plain
+ * or packed expert weights (xshare_pack_experts), with optional per-kernel
+ * events; xshare_stack_forward and its CUDA-graph form (L layers under one
+ * global budget); a bounded-wait self-test; strings.
  */
 #ifndef XSHARE_H
 #define XSHARE_H
