@@ -25,6 +25,8 @@ constexpr int kRows = 128, kCols = 64, kTile = kRows * kCols * 2;
 // W0 (and W1 if given) [n][M][K] bf16 -> P, `per` tiles per block (1 or 2).
 __global__ void __launch_bounds__(256) pack_kernel(const uint4 *__restrict__ W0, const uint4 *__restrict__ W1,
                                                    uint8_t *__restrict__ P, int n, int M, int K) {
+  pdl_wait();  // the weights may still be being written by the work before this call
+  pdl_trigger();
   const int per = W1 ? 2 : 1;
   const int MT = M / kRows, KI = K / kCols, KC = K / 8;   // 16-byte chunks per row
   const long long chunks = static_cast<long long>(n) * M * KC;
