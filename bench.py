@@ -78,6 +78,8 @@ def parse_args(argv=None):
                     help="stack budget K (default: layers x the per-layer budget)")
     ap.add_argument("--unpacked", action="store_true",
                     help="read the expert weights as plain [N, F, d] matrices instead of packed tiles")
+    ap.add_argument("--e2e-eager", action="store_true",
+                    help="end-to-end steps as eager calls instead of CUDA-graph replays")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--seed", type=int, default=0)
     return ap.parse_args(argv)
@@ -396,11 +398,34 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
     x_in = torch.empty(w.B, w.d, dtype=torch.bfloat16, device=dev)
     st_dev = torch.zeros(X.STATS_WORDS, dtype=torch.int32, device=dev)
 
-    def e2e_step(i):
+    def e2e_body(i):
         x_in.copy_(x_pin[i % N_ROTATE], non_blocking=True)
         forward(x_in, st_dev)
         y_pin.copy_(y, non_blocking=True)
         st_pin.copy_(st_dev, non_blocking=True)
+
+    # By default each step replays a CUDA graph of the copy in, the forward
+    # (the library's calls are capture-safe) and the copies out, one graph per
+    # rotating input buffer, as a decode server would; --e2e-eager issues the
+    # calls one by one every step.
+    graphs = []
+    if not args.e2e_eager:
+        for i in range(Wm):
+            e2e_body(i)
+        torch.cuda.synchronize()
+        for i in range(N_ROTATE):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, capture_error_mode="thread_local"):
+                e2e_body(i)
+            graphs.append(g)
+        torch.cuda.synchronize()
+        stream = torch.cuda.current_stream()
+
+    def e2e_step(i):
+        if graphs:
+            graphs[i % N_ROTATE].replay()
+        else:
+            e2e_body(i)
         stream.synchronize()
 
     for i in range(Wm):
@@ -471,6 +496,8 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
             "unit": "tokens/s",
             "h2d_bytes_per_step": w.B * w.d * 2,
             "d2h_bytes_per_step": w.B * w.d * 2 + X.STATS_WORDS * 4,
+            "method": "CUDA-graph replay of copy in + xshare forward + copies out, host sync every step"
+                      if graphs else "eager calls, host sync every step",
         },
         "gpu_launches": launches_per_step * K,
     }
