@@ -53,6 +53,10 @@ struct Cfg {
   static constexpr int kNumA = kGateUp ? 2 : 1;          // weight tiles per stage
   static constexpr int kStages = kGateUp ? 3 : 6;   // measured best on GB300 (3, 4 and 2; 4, 5 and 6)
   static constexpr int kStageBytes = kNumA * kTileBytes + kTileBytes;
+  // Weights fetched before pdl_wait(): the ring's first stages, then an L2
+  // prefetch of the weights after them, 64 KB per CTA (measured best on GB300
+  // among 0 to 256 KB; more competes with the kernel before for HBM).
+  static constexpr int kL2Prefetch = 64 * 1024;
   static constexpr int kAccCols = kGateUp ? 256 : 128;   // TMEM columns per buffer
   static constexpr int kTmemCols = 2 * kAccCols;
   static constexpr int kBarOffset = kStages * kStageBytes;
@@ -122,18 +126,23 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
   volatile int *s_flag = reinterpret_cast<volatile int *>(tmem_slot + 2);
 
-  pdl_wait();
-  pdl_trigger();
+  // The routing kernels that wrote meta and tiles finished before this grid
+  // could start (every kernel of the chain calls pdl_trigger() only after its
+  // own pdl_wait()), so they may be read here through L2 before pdl_wait();
+  // only the token operand and the outputs depend on the kernel just before.
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n_tiles = p.meta->n_tiles;
+  const int n_tiles = __ldcg(&p.meta->n_tiles);
   const int MT = p.M / kBM, KI = p.K / kBK;
   Range rg;
   rg.KI = KI;
   rg.I = static_cast<long long>(n_tiles) * MT * KI;
-  if (rg.I == 0) return;
   const long long want = (rg.I + kMinItersPerCta - 1) / kMinItersPerCta;
   rg.G = static_cast<int>(want < p.grid ? want : p.grid);
-  if (static_cast<int>(blockIdx.x) >= rg.G) return;
+  if (rg.I == 0 || static_cast<int>(blockIdx.x) >= rg.G) {
+    pdl_wait();
+    pdl_trigger();
+    return;
+  }
   const int cta = blockIdx.x;
   const long long it_begin = rg.begin(cta), it_end = rg.begin(cta + 1);
 
@@ -168,57 +177,125 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
+  // Where unit u's operands come from.
+  struct Src {
+    int ntok, row0, bsel, arow;
+    uint32_t tx;
+    const CUtensorMap *mA0, *mA1;
+    const uint8_t *pblk;   // packed: the unit's blocks are consecutive, one per K step
+  };
+  // Before pdl_wait() the tile is read through L2 only; after it, with a
+  // plain load that also leaves it in L1 for the MMA and epilogue warps.
+  auto src_of = [&](long long u, bool early) {
+    const int4 *tp = reinterpret_cast<const int4 *>(p.tiles) + u / MT;
+    const int4 t4 = early ? __ldcg(tp) : *tp;
+    Src r;
+    r.ntok = t4.z;
+    r.row0 = t4.y;
+    const int mt = static_cast<int>(u % MT);
+    // One box of 16, 32, 64 or 128 token rows covers the tile's tokens.
+    r.bsel = r.ntok <= 16 ? 0 : r.ntok <= 32 ? 1 : r.ntok <= 64 ? 2 : 3;
+    r.tx = C::kNumA * kTileBytes + (kBoxTok << r.bsel) * kBK * 2;
+    const bool routed = t4.x < p.n_routed;
+    r.mA0 = routed ? &p.tmA0 : &p.tmS0;
+    r.mA1 = routed ? &p.tmA1 : &p.tmS1;
+    const int e_local = routed ? t4.x : t4.x - p.n_routed;
+    r.arow = e_local * p.M + mt * kBM;
+    r.pblk = p.pk ? (routed ? p.pk : p.pk_shared) +
+                        ((static_cast<size_t>(e_local) * MT + mt) * KI) * (C::kNumA * kTileBytes)
+                  : nullptr;
+    return r;
+  };
+  auto load_weights = [&](const Src &r, int kk, uint32_t sA, uint32_t bar, uint64_t pol) {
+    if (r.pblk) {
+      bulk_load(sA, r.pblk + static_cast<size_t>(kk) * (C::kNumA * kTileBytes), C::kNumA * kTileBytes,
+                bar, pol);
+    } else {
+      tma_load_2d(sA, r.mA0, bar, kk * kBK, r.arow, pol);
+      if (kGateUp) tma_load_2d(sA + kTileBytes, r.mA1, bar, kk * kBK, r.arow, pol);
+    }
+  };
+  const bool producer = warp == 0 && lane == 0;
+  const int n_pre = (it_end - it_begin) < C::kStages ? static_cast<int>(it_end - it_begin) : C::kStages;
+  // The producer walks its K steps with a cursor (unit u, step kk of it) and
+  // re-reads the unit's source only when u changes.
+  struct Cursor {
+    long long u;
+    int kk;
+    bool fresh;
+  };
+  const Cursor c_begin{it_begin / KI, static_cast<int>(it_begin % KI), true};
+  auto advance = [&](Cursor &c) {
+    if (++c.kk == KI) {
+      c.kk = 0;
+      ++c.u;
+      c.fresh = true;
+    }
+  };
+  auto source = [&](Cursor &c, Src &r, bool early) {
+    if (c.fresh) {
+      r = src_of(c.u, early);
+      c.fresh = false;
+    }
+  };
+  uint64_t pol_w = 0, pol_x = 0;
+  if (producer) {
+    // Every stage is free at the start: fill the ring with weights and warm L2
+    // with the weights that follow.
+    pol_w = policy_evict_first();
+    pol_x = policy_evict_last();
+    Cursor c = c_begin;
+    Src r{};
+    for (int i = 0; i < n_pre; ++i, advance(c)) {
+      source(c, r, true);
+      mbar_arrive_expect_tx(full_bar(i), r.tx);
+      load_weights(r, c.kk, sbase + i * C::kStageBytes, full_bar(i), pol_w);
+    }
+    if (p.pk) {
+      const long long n_pf = C::kL2Prefetch / (C::kNumA * kTileBytes);
+      for (long long it = it_begin + n_pre; it < it_end && it < it_begin + n_pre + n_pf; ++it, advance(c)) {
+        source(c, r, true);
+        bulk_prefetch_l2(r.pblk + static_cast<size_t>(c.kk) * (C::kNumA * kTileBytes),
+                         C::kNumA * kTileBytes);
+      }
+    }
+  }
+  pdl_wait();
+  pdl_trigger();
+
   if (warp == 0) {
     // ------------------------------------------------ TMA producer
     if (lane == 0) {
-      const uint64_t pol_w = policy_evict_first(), pol_x = policy_evict_last();
-      int stage = 0;
-      uint32_t phase = 0;
       uint32_t issued_mask = 0, issued_phase = 0;
+      Cursor c = c_begin;
+      Src r{};
+      // Token operand of the stages filled above.
+      for (int i = 0; i < n_pre; ++i, advance(c)) {
+        source(c, r, false);
+        tma_load_2d(sbase + i * C::kStageBytes + C::kNumA * kTileBytes, &p.tmB[r.bsel], full_bar(i),
+                    c.kk * kBK, r.row0, pol_x);
+        issued_mask |= 1u << i;
+      }
+      int stage = static_cast<int>(n_pre % C::kStages);
+      uint32_t phase = n_pre == C::kStages ? 1u : 0u;
       bool ok = true;
-      for (long long it = it_begin; ok && it < it_end;) {
-        const long long u = it / KI;
-        const int k0 = static_cast<int>(it - u * KI);
-        const int k1 = static_cast<int>(k0 + (it_end - it) < KI ? k0 + (it_end - it) : KI);
-        const Tile tl = p.tiles[u / MT];
-        const int mt = static_cast<int>(u % MT);
-        // One box of 16, 32, 64 or 128 token rows covers the tile's tokens.
-        const int bsel = tl.ntok <= 16 ? 0 : tl.ntok <= 32 ? 1 : tl.ntok <= 64 ? 2 : 3;
-        const uint32_t tx = C::kNumA * kTileBytes + (kBoxTok << bsel) * kBK * 2;
-        const bool routed = tl.expert < p.n_routed;
-        const CUtensorMap *mA0 = routed ? &p.tmA0 : &p.tmS0;
-        const CUtensorMap *mA1 = routed ? &p.tmA1 : &p.tmS1;
-        const int e_local = routed ? tl.expert : tl.expert - p.n_routed;
-        const int arow = e_local * p.M + mt * kBM;
-        // Packed weights: the unit's blocks are consecutive, one per K step.
-        const uint8_t *pblk =
-            p.pk ? (routed ? p.pk : p.pk_shared) +
-                       ((static_cast<size_t>(e_local) * MT + mt) * KI) * (C::kNumA * kTileBytes)
-                 : nullptr;
-        for (int kk = k0; kk < k1; ++kk) {
-          if (!mbar_wait(empty_bar(stage), phase ^ 1u, kWaitNs, abort_flag)) {
-            ok = false;
-            break;
-          }
-          const uint32_t sA = sbase + stage * C::kStageBytes;
-          const uint32_t sB = sA + C::kNumA * kTileBytes;
-          mbar_arrive_expect_tx(full_bar(stage), tx);
-          if (pblk) {
-            bulk_load(sA, pblk + static_cast<size_t>(kk) * (C::kNumA * kTileBytes), C::kNumA * kTileBytes,
-                      full_bar(stage), pol_w);
-          } else {
-            tma_load_2d(sA, mA0, full_bar(stage), kk * kBK, arow, pol_w);
-            if (kGateUp) tma_load_2d(sA + kTileBytes, mA1, full_bar(stage), kk * kBK, arow, pol_w);
-          }
-          tma_load_2d(sB, &p.tmB[bsel], full_bar(stage), kk * kBK, tl.row0, pol_x);
-          issued_mask |= 1u << stage;
-          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-          if (++stage == C::kStages) {
-            stage = 0;
-            phase ^= 1u;
-          }
+      for (long long it = it_begin + n_pre; it < it_end; ++it, advance(c)) {
+        source(c, r, false);
+        const int kk = c.kk;
+        if (!mbar_wait(empty_bar(stage), phase ^ 1u, kWaitNs, abort_flag)) {
+          ok = false;
+          break;
         }
-        it += k1 - k0;
+        const uint32_t sA = sbase + stage * C::kStageBytes;
+        mbar_arrive_expect_tx(full_bar(stage), r.tx);
+        load_weights(r, kk, sA, full_bar(stage), pol_w);
+        tma_load_2d(sA + C::kNumA * kTileBytes, &p.tmB[r.bsel], full_bar(stage), kk * kBK, r.row0, pol_x);
+        issued_mask |= 1u << stage;
+        issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+        if (++stage == C::kStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
       }
       if (!ok) {
         set_status(p, XS_DEV_TIMEOUT);

@@ -11,11 +11,15 @@
 namespace xs {
 
 // Programmatic dependent launch.  Every kernel of the library is launched
-// with programmatic stream serialization and starts with pdl_wait(), which
-// returns once all work before it in the stream has completed and is
-// visible; it then calls pdl_trigger() so that the next kernel's CTAs may be
-// scheduled while this one runs (they block in their own pdl_wait()).  A CTA
-// touches no global memory before pdl_wait().
+// with programmatic stream serialization and calls pdl_wait(), which returns
+// once all work before it in the stream has completed and is visible, and
+// only after that pdl_trigger(), so that the next kernel's CTAs may be
+// scheduled while this one runs (they block in their own pdl_wait()).  Every
+// CTA waits before it exits.  Hence when a CTA of kernel n starts, kernel
+// n - 2 and everything before it have completed: the FFN kernels read the
+// routing results (written two or more launches earlier) and start their
+// weight loads before pdl_wait(); every other access to global memory, in
+// every kernel, comes after it.
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
