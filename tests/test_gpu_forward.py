@@ -273,11 +273,17 @@ def test_forward_shared_experts_full_size_sampled(X):
 
 
 # ---- router logits on either path (CUDA cores below 64 tokens, tensor cores from 64) ----
+# Below 64 tokens: one or two token blocks, ragged expert blocks (N = 100),
+# every cluster split of d (d = 128: 1; 512: 4; 2048 and 7168: 8 or 4) and the
+# unsplit grid of N = 1024.
 @pytest.mark.parametrize("w", [
+    W.TINY.with_(B=1, budget=8), W.TINY.with_(B=33), W.TINY.with_(N=100, B=40),
+    W.TINY.with_(d=128, F=128, B=20, budget=8), W.TINY.with_(N=1024, k=16, budget=64, B=16),
     W.TINY.with_(B=63), W.TINY.with_(B=64), W.TINY.with_(B=65, budget=16),
-    W.OLMOE.with_(B=200), W.QWEN3.with_(B=1000, tokens_per_request=8),
-    W.DSR1.with_(B=256, budget=40),
-], ids=lambda w: f"{w.name}-B{w.B}")
+    W.OLMOE.with_(B=8, budget=16), W.OLMOE.with_(B=200), W.QWEN3.with_(B=48),
+    W.QWEN3.with_(B=1000, tokens_per_request=8),
+    W.DSR1, W.DSR1.with_(B=256, budget=40),
+], ids=lambda w: f"{w.name}-N{w.N}-d{w.d}-B{w.B}")
 def test_router_scores_both_paths(X, w):
     """The dense scores from the router and softmax are within P_RTOL of the
     oracle's (fp64 logits, fp32 softmax), elementwise, and repeat bit for bit."""
