@@ -186,7 +186,7 @@ extern "C" int xshare_route(const float *scores, int B, int N, int k, int budget
   a.offsets_out = expert_offsets;
   a.perm_out = perm;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (cudaMemsetAsync(a.done, 0, 2 * sizeof(int32_t), s) != cudaSuccess) return XS_ERR_CUDA;
+  if (cudaMemsetAsync(a.done, 0, 3 * sizeof(int32_t), s) != cudaSuccess) return XS_ERR_CUDA;
   return launch_route(a, s) == cudaSuccess ? XS_OK : XS_ERR_CUDA;
 }
 

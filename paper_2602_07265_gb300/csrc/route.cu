@@ -149,6 +149,22 @@ __device__ __forceinline__ void lane_load(LaneList<Q> &L, int j0, int n, int lan
   }
 }
 
+// Moves each lane's best candidate to slot 0 (enough for a single take).
+template <int Q>
+__device__ __forceinline__ void lane_head(LaneList<Q> &L) {
+#pragma unroll
+  for (int q = 1; q < Q; ++q) {
+    if (before(L.key[q], L.idx[q], L.key[0], L.idx[0])) {
+      const uint32_t tk = L.key[0];
+      L.key[0] = L.key[q];
+      L.key[q] = tk;
+      const int ti = L.idx[0];
+      L.idx[0] = L.idx[q];
+      L.idx[q] = ti;
+    }
+  }
+}
+
 // Exclusive block-wide scan of three ints per thread; returns the totals.
 __device__ __forceinline__ void block_scan3(int (&v)[3], int (&tot)[3], int *s_tmp /*[32][3]*/) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
@@ -213,10 +229,9 @@ __device__ __forceinline__ void block_scan3(int (&v)[3], int (&tot)[3], int *s_t
 
 __device__ __forceinline__ int chunk_count(int B) { return (B + kChunk - 1) / kChunk; }
 
-// Selected set statistics: |S|, plain top-k union, max group load.
-__device__ __forceinline__ void selection_stats(const RouteArgs &a, const uint8_t *s_mask,
-                                                const uint8_t *s_union, int *s_gl, int &nsel,
-                                                int &n_union, int &maxload) {
+// Selected set statistics: |S| and the max group load.
+__device__ __forceinline__ void selection_stats(const RouteArgs &a, const uint8_t *s_mask, int *s_gl,
+                                                int &nsel, int &maxload) {
   const int tid = threadIdx.x, N = a.N;
   const int G = a.G >= 1 ? a.G : 1, size = N / G;
   for (int g = tid; g < G; g += blockDim.x) s_gl[g] = 0;
@@ -224,7 +239,6 @@ __device__ __forceinline__ void selection_stats(const RouteArgs &a, const uint8_
   for (int j = tid; j < N; j += blockDim.x)
     if (s_mask[j]) atomicAdd(&s_gl[j / size], 1);
   nsel = __syncthreads_count(tid < N && s_mask[tid]);
-  n_union = __syncthreads_count(tid < N && s_union[tid]);
   int best = 0;
   for (int g = tid; g < G; g += blockDim.x) best = max(best, s_gl[g]);
   best = __reduce_max_sync(kFull, best);
@@ -384,23 +398,108 @@ __device__ void build_permutation(const RouteArgs &a, PermSmem sm) {
     }
   }
   if (tid == 0) {
-    Meta m = *a.meta;
-    m.n_pairs = sm.scal[1];  // == B * kp unless scores were non-finite
-    m.n_tiles = sm.scal[2] + a.n_shared * ((B + kTileTok - 1) / kTileTok);
-    m.n_used = sm.scal[3];
-    m.n_rows = sm.scal[1] + a.n_shared * B;
-    *a.meta = m;
+    // Field by field: union_topk belongs to the union CTAs (score_kernel).
+    Meta *m = a.meta;
+    m->n_pairs = sm.scal[1];  // == B * kp unless scores were non-finite
+    m->n_tiles = sm.scal[2] + a.n_shared * ((B + kTileTok - 1) / kTileTok);
+    m->n_used = sm.scal[3];
+    m->n_rows = sm.scal[1] + a.n_shared * B;
     if (a.stats) {
-      xs_stats st;
-      st.n_selected = m.n_selected;
-      st.n_used = m.n_used;
-      st.union_topk = m.union_topk;
-      st.max_group_load = m.max_group_load;
-      st.n_pairs = m.n_pairs;
-      st.status = m.status;
-      st.reserved[0] = st.reserved[1] = 0;
-      *a.stats = st;
+      xs_stats *st = a.stats;
+      st->n_selected = m->n_selected;
+      st->n_used = sm.scal[3];
+      st->max_group_load = m->max_group_load;
+      st->n_pairs = sm.scal[1];
+      st->status = m->status;
+      st->reserved[0] = st->reserved[1] = 0;
     }
+  }
+}
+
+// Token t's dense scores (a2) in vals[q] = p[t, lane + 32 q] (0 past N): the
+// softmax of its logits (written to a.p when write_p), or the given scores.
+template <int kQ>
+__device__ __forceinline__ void token_scores(const RouteArgs &a, int t, int lane, float (&vals)[kQ],
+                                             bool write_p) {
+  const int N = a.N;
+  if (a.logits != nullptr) {
+    const float *hrow = a.logits + (size_t)t * N;
+    float mx = -INFINITY;
+#pragma unroll
+    for (int q = 0; q < kQ; ++q) {
+      const int j = lane + 32 * q;
+      vals[q] = (j < N) ? hrow[j] : -INFINITY;
+      mx = fmaxf(mx, vals[q]);
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, o));
+    float sum = 0.f;
+#pragma unroll
+    for (int q = 0; q < kQ; ++q) {
+      vals[q] = (lane + 32 * q < N) ? expf(vals[q] - mx) : 0.f;
+      sum = __fadd_rn(sum, vals[q]);
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) sum = __fadd_rn(sum, __shfl_xor_sync(kFull, sum, o));
+#pragma unroll
+    for (int q = 0; q < kQ; ++q) {
+      const int j = lane + 32 * q;
+      if (j < N) {
+        vals[q] = __fdiv_rn(vals[q], sum);
+        if (write_p) a.p[(size_t)t * N + j] = vals[q];
+      }
+    }
+  } else {
+#pragma unroll
+    for (int q = 0; q < kQ; ++q) {
+      const int j = lane + 32 * q;
+      vals[q] = (j < N) ? a.p[(size_t)t * N + j] : 0.f;
+    }
+  }
+}
+
+// The plain top-k union (a statistic): CTA C + c ranks the k best experts of
+// every token of chunk c over E, concurrently with the selection CTAs, and
+// the last of these CTAs to finish counts the union and writes union_topk.
+template <int kQ>
+__device__ __noinline__ void union_cta(const RouteArgs &a, uint8_t *s_union, int32_t *s_flag) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarps = blockDim.x >> 5;
+  const int B = a.B, N = a.N, k = a.k;
+  const int C = chunk_count(B), c = blockIdx.x - C;
+  const int t0 = c * kChunk, nt = min(kChunk, B - t0);
+  for (int j = tid; j < N; j += blockDim.x) s_union[j] = 0;
+  __syncthreads();
+  for (int w = warp; w < nt; w += nwarps) {
+    float vals[kQ];
+    token_scores<kQ>(a, t0 + w, lane, vals, false);
+    LaneList<kQ> L;
+    lane_load<kQ>(L, 0, N, lane, [&](int q, int) { return vals[q]; }, [](int, int) { return true; });
+    lane_sort<kQ>(L);
+    lane_take<kQ>(L, k, [&](int, int id, float) {
+      if (lane == 0) s_union[id] = 1;
+    });
+  }
+  __syncthreads();
+  if (C > 1) {
+    uint8_t *marks = a.chunk_marks + (size_t)c * 2 * N + N;
+    for (int j = tid; j < N; j += blockDim.x) marks[j] = s_union[j];
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) *s_flag = (atomicAdd(&a.done[2], 1) == C - 1) ? 1 : 0;
+    __syncthreads();
+    if (!*s_flag) return;
+    __threadfence();
+    for (int j = tid; j < N; j += blockDim.x) {
+      uint8_t u = 0;
+      for (int cc = 0; cc < C; ++cc) u |= __ldcg(a.chunk_marks + (size_t)cc * 2 * N + N + j);
+      s_union[j] = u;
+    }
+    __syncthreads();
+  }
+  const int n_union = __syncthreads_count(tid < N && s_union[tid]);
+  if (tid == 0) {
+    a.meta->union_topk = n_union;
+    if (a.stats) a.stats->union_topk = n_union;
   }
 }
 
@@ -409,7 +508,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   extern __shared__ float ps[];         // [32][N] scores of the chunk's tokens (+ [32][N] ints)
   __shared__ uint8_t s_mask[kMaxN];     // S (selection step)
   __shared__ uint8_t s_base[kMaxN];     // chunk marks: S_0 (or S_r for HIER); merged later
-  __shared__ uint8_t s_union[kMaxN];    // chunk marks: plain top-k union; merged later
+  __shared__ uint8_t s_union[kMaxN];    // union CTAs: plain top-k union marks
   __shared__ float s_col[kMaxN];
   __shared__ int32_t s_gl[kMaxN + 1];
   __shared__ int32_t s_top[kChunk][kMaxK];
@@ -425,17 +524,20 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   const int nwarps = blockDim.x >> 5;
   const int B = a.B, N = a.N, k = a.k;
   const int C = chunk_count(B), c = blockIdx.x;
+  if (c >= C) {  // CTAs C .. 2C - 1 count the plain top-k union
+    union_cta<kQ>(a, s_union, s_scal);
+    return;
+  }
   const int t0 = c * kChunk, nt = min(kChunk, B - t0);
-  const int kk = max(k, a.k0);
+  // Ranking depth the selection needs: the warm-up top-k0, and the token's
+  // top-k for Sec. 2.2's gating values when the column scores are sparse.
+  const int kk = a.sparse ? max(k, a.k0) : a.k0;
   const bool hier = a.mode == XS_MODE_HIER;
   // HIER requests that lie inside one chunk are selected here (Algorithm 3);
   // otherwise the selection step does it from the full score matrix.
   const bool hier_here = hier && a.T <= kChunk && kChunk % a.T == 0;
 
-  for (int j = tid; j < N; j += blockDim.x) {
-    s_base[j] = 0;
-    s_union[j] = 0;
-  }
+  for (int j = tid; j < N; j += blockDim.x) s_base[j] = 0;
   if (a.zero_words != nullptr)
     for (int i = c * blockDim.x + tid; i < a.zero_count; i += C * blockDim.x) a.zero_words[i] = 0;
   __syncthreads();
@@ -449,52 +551,23 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
     }
     const int t = t0 + w;
     float vals[kQ];
-    if (a.logits != nullptr) {
-      const float *hrow = a.logits + (size_t)t * N;
-      float mx = -INFINITY;
+    token_scores<kQ>(a, t, lane, vals, true);
 #pragma unroll
-      for (int q = 0; q < kQ; ++q) {
-        const int j = lane + 32 * q;
-        vals[q] = (j < N) ? hrow[j] : -INFINITY;
-        mx = fmaxf(mx, vals[q]);
-      }
-#pragma unroll
-      for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, o));
-      float sum = 0.f;
-#pragma unroll
-      for (int q = 0; q < kQ; ++q) {
-        vals[q] = (lane + 32 * q < N) ? expf(vals[q] - mx) : 0.f;
-        sum = __fadd_rn(sum, vals[q]);
-      }
-#pragma unroll
-      for (int o = 16; o; o >>= 1) sum = __fadd_rn(sum, __shfl_xor_sync(kFull, sum, o));
-#pragma unroll
-      for (int q = 0; q < kQ; ++q) {
-        const int j = lane + 32 * q;
-        if (j < N) {
-          vals[q] = __fdiv_rn(vals[q], sum);
-          a.p[(size_t)t * N + j] = vals[q];
-          prow_s[j] = vals[q];
-        }
-      }
-    } else {
-#pragma unroll
-      for (int q = 0; q < kQ; ++q) {
-        const int j = lane + 32 * q;
-        vals[q] = (j < N) ? a.p[(size_t)t * N + j] : 0.f;
-        if (j < N) prow_s[j] = vals[q];
-      }
-    }
+    for (int q = 0; q < kQ; ++q)
+      if (lane + 32 * q < N) prow_s[lane + 32 * q] = vals[q];
+    if (kk == 0) continue;
     LaneList<kQ> L;
     lane_load<kQ>(L, 0, N, lane, [&](int q, int) { return vals[q]; },
                   [](int, int) { return true; });
-    lane_sort<kQ>(L);
+    if (kk == 1)
+      lane_head<kQ>(L);
+    else
+      lane_sort<kQ>(L);
     int32_t *top = a.toptok + (size_t)t * kMaxK;
     int my_id = -1;  // sparse scores: lane s keeps slot s of the token's top-k
     float my_v = 0.f, D = 0.f;
     lane_take<kQ>(L, kk, [&](int r, int id, float v) {
       if (lane == 0) {
-        if (r < k) s_union[id] = 1;
         if (r < a.k0) {
           s_top[w][r] = id;
           if (hier)
@@ -580,10 +653,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   __syncthreads();
   if (C > 1) {
     uint8_t *marks = a.chunk_marks + (size_t)c * 2 * N;
-    for (int j = tid; j < N; j += blockDim.x) {
-      marks[j] = s_base[j];
-      marks[N + j] = s_union[j];
-    }
+    for (int j = tid; j < N; j += blockDim.x) marks[j] = s_base[j];
 
     // ---- the last CTA to finish runs the selection ----
     __threadfence();
@@ -595,16 +665,13 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
 
     for (int j = tid; j < N; j += blockDim.x) {
       float acc = 0.f;
-      uint8_t b = 0, u = 0;
+      uint8_t b = 0;
       for (int cc = 0; cc < C; ++cc) {
         acc = __fadd_rn(acc, __ldcg(a.chunk_col + (size_t)cc * N + j));
-        const uint8_t *m = a.chunk_marks + (size_t)cc * 2 * N;
-        b |= __ldcg(m + j);
-        u |= __ldcg(m + N + j);
+        b |= __ldcg(a.chunk_marks + (size_t)cc * 2 * N + j);
       }
       s_col[j] = acc;
       s_base[j] = b;
-      s_union[j] = u;
     }
   }
   __syncthreads();
@@ -729,26 +796,24 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   }
   __syncthreads();
 
-  int nsel, n_union, maxload;
+  int nsel, maxload;
   if (tid == 0) s_gl[kMaxN] = 0;
-  selection_stats(a, s_mask, s_union, s_gl, nsel, n_union, maxload);
+  selection_stats(a, s_mask, s_gl, nsel, maxload);
   for (int j = tid; j < N; j += blockDim.x) a.mask[j] = s_mask[j];
   int rstat = 0;  // the router's status, if it reports one
   for (int i = tid; i < a.router_ctas; i += blockDim.x) rstat = max(rstat, __ldcg(a.router_status + i));
   rstat = __syncthreads_or(rstat);
   if (tid == 0) {
-    Meta m;
-    for (int i = 0; i < 7; ++i) m.pad[i] = 0;
-    m.n_pairs = 0;
-    m.n_tiles = 0;
-    m.n_rows = 0;
-    m.kprime = min(k, nsel);
-    m.n_selected = nsel;
-    m.n_used = 0;
-    m.union_topk = n_union;
-    m.max_group_load = maxload;
-    m.status = rstat ? XS_DEV_TIMEOUT : XS_DEV_OK;
-    *a.meta = m;
+    // Field by field: union_topk belongs to the union CTAs.
+    Meta *m = a.meta;
+    m->n_pairs = 0;
+    m->n_tiles = 0;
+    m->n_rows = 0;
+    m->kprime = min(k, nsel);
+    m->n_selected = nsel;
+    m->n_used = 0;
+    m->max_group_load = maxload;
+    m->status = rstat ? XS_DEV_TIMEOUT : XS_DEV_OK;
   }
   if (!a.fuse_refine) return;
   // Small batches: refinement and permutation in this CTA too (no second
@@ -831,7 +896,7 @@ __global__ void __launch_bounds__(kRtWarps * 32) router_logits_kernel(
   __shared__ float red[kRtWarps][kRtOut];
   pdl_wait();
   pdl_trigger();
-  if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x < 2) done[threadIdx.x] = 0;
+  if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x < 3) done[threadIdx.x] = 0;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int e0 = blockIdx.x * kRtExp, t0 = blockIdx.y * kRtTok;
   const int d4 = d / 4;
@@ -975,7 +1040,7 @@ cudaError_t launch_route_q(const RouteArgs &a, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(score_kernel<kQ>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, dyn1);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(score_kernel<kQ>, dim3(C), dim3(kRouteThreads), (size_t)dyn1, s, b);
+  e = launch_pdl(score_kernel<kQ>, dim3(2 * C), dim3(kRouteThreads), (size_t)dyn1, s, b);
   if (e != cudaSuccess) return e;
   if (b.fuse_refine) {
     if (a.events != nullptr) e = cudaEventRecord(reinterpret_cast<cudaEvent_t>(a.events[0]), s);

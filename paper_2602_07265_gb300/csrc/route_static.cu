@@ -123,9 +123,9 @@ extern "C" int xshare_route_static(const float *scores, int B, int N, int k, int
   a.done = reinterpret_cast<int32_t *>(base + kOffDone);
   a.zero_words = nullptr;
   a.zero_count = 0;
-  // The two arrival counters must start at zero; every other scratch word is
+  // The three arrival counters must start at zero; every other scratch word is
   // written before it is read.
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (cudaMemsetAsync(a.done, 0, 2 * sizeof(int32_t), s) != cudaSuccess) return XS_ERR_CUDA;
+  if (cudaMemsetAsync(a.done, 0, 3 * sizeof(int32_t), s) != cudaSuccess) return XS_ERR_CUDA;
   return launch_route(a, s) == cudaSuccess ? XS_OK : XS_ERR_CUDA;
 }
