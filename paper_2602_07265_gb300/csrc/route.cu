@@ -247,24 +247,52 @@ __device__ __forceinline__ void selection_stats(const RouteArgs &a, const uint8_
   maxload = s_gl[kMaxN];
 }
 
+// The experts of S in ascending order into s_list; returns |S|.  One thread
+// per expert (blockDim >= N); s_wc: [32] scratch.
+__device__ __forceinline__ int compact_selected(const uint8_t *s_mask, int N, int32_t *s_list,
+                                                int *s_wc) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
+  const bool m = tid < N && s_mask[tid] != 0;
+  const unsigned b = __ballot_sync(kFull, m);
+  if (lane == 0) s_wc[warp] = __popc(b);
+  __syncthreads();
+  int base = 0, total = 0;
+  for (int w = 0; w < nw; ++w) {
+    const int c = s_wc[w];
+    base += (w < warp) ? c : 0;
+    total += c;
+  }
+  if (m) s_list[base + __popc(b & ((1u << lane) - 1u))] = tid;
+  __syncthreads();
+  return total;
+}
+
+static_assert(kRouteThreads >= kMaxN, "compact_selected takes one thread per expert");
+
 // Per token t in [t_begin, t_end), one warp each: Top k'(G_t, S) with the
-// renormalised weights (a6); row(t) points at the token's scores.
-template <int kQ, class Row>
-__device__ __forceinline__ void refine_tokens(const RouteArgs &a, const uint8_t *s_mask,
-                                              int t_begin, int t_end, int kp, Row row,
-                                              int32_t *ids_s = nullptr) {
+// renormalised weights (a6); row(t) points at the token's scores.  Lane l
+// ranks the experts s_list[l + 32 q] of S (q < Q, Q * 32 >= |S|).
+template <int Q, class Row>
+__device__ __forceinline__ void refine_tokens_q(const RouteArgs &a, const int32_t *s_list, int nS,
+                                                int t_begin, int t_end, int kp, Row row,
+                                                int32_t *ids_s) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
-  const int N = a.N, k = a.k;
+  const int k = a.k;
   for (int t = t_begin + warp; t < t_end; t += nwarps) {
     const float *prow = row(t);
-    LaneList<kQ> L;
-    lane_load<kQ>(L, 0, N, lane, [&](int, int j) { return prow[j]; },
-                  [&](int, int j) { return s_mask[j] != 0; });
-    lane_sort<kQ>(L);
+    LaneList<Q> L;
+#pragma unroll
+    for (int q = 0; q < Q; ++q) {
+      const int i = lane + 32 * q;
+      const int e = i < nS ? s_list[i] : 0;
+      L.idx[q] = e;
+      L.key[q] = i < nS ? score_key(prow[e]) : 0u;
+    }
+    lane_sort<Q>(L);
     int my_id = -1;  // lane s keeps slot s
     float my_v = 0.f;
     float D = 0.f;
-    const int got = lane_take<kQ>(L, kp, [&](int r, int id, float v) {
+    const int got = lane_take<Q>(L, kp, [&](int r, int id, float v) {
       if (lane == r) {
         my_id = id;
         my_v = v;
@@ -278,6 +306,60 @@ __device__ __forceinline__ void refine_tokens(const RouteArgs &a, const uint8_t 
       if (ids_s) ids_s[(t - t_begin) * k + lane] = (lane < got) ? my_id : -1;
       a.w[(size_t)t * k + lane] = wv;
     }
+  }
+}
+
+// The same over all N experts with the mask (lane l: experts l + 32 q).
+template <int kQ, class Row>
+__device__ __forceinline__ void refine_tokens_masked(const RouteArgs &a, const uint8_t *s_mask,
+                                                     int t_begin, int t_end, int kp, Row row,
+                                                     int32_t *ids_s) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  const int N = a.N, k = a.k;
+  for (int t = t_begin + warp; t < t_end; t += nwarps) {
+    const float *prow = row(t);
+    LaneList<kQ> L;
+    lane_load<kQ>(L, 0, N, lane, [&](int, int j) { return prow[j]; },
+                  [&](int, int j) { return s_mask[j] != 0; });
+    lane_sort<kQ>(L);
+    int my_id = -1;
+    float my_v = 0.f;
+    float D = 0.f;
+    const int got = lane_take<kQ>(L, kp, [&](int r, int id, float v) {
+      if (lane == r) {
+        my_id = id;
+        my_v = v;
+      }
+      D = __fadd_rn(D, v);
+    });
+    if (lane < k) {
+      float wv = 0.f;
+      if (lane < got) wv = (D > 0.f) ? __fdiv_rn(my_v, D) : __fdiv_rn(1.f, (float)got);
+      a.ids[(size_t)t * k + lane] = (lane < got) ? my_id : -1;
+      if (ids_s) ids_s[(t - t_begin) * k + lane] = (lane < got) ? my_id : -1;
+      a.w[(size_t)t * k + lane] = wv;
+    }
+  }
+}
+
+// Refinement of tokens [t_begin, t_end) against S (|S| = nS, the mask in
+// s_mask).  When S fits a shorter lane list than all N experts need, its
+// experts are first compacted into s_list (then [kMaxN] scratch, s_wc [32]);
+// either way the candidates and their order are the same.  Every thread of
+// the block calls it with the same nS.
+template <int kQ, class Row>
+__device__ __forceinline__ void refine_tokens(const RouteArgs &a, const uint8_t *s_mask, int nS,
+                                              int32_t *s_list, int *s_wc, int t_begin, int t_end,
+                                              int kp, Row row, int32_t *ids_s = nullptr) {
+  const int nq = (nS + 31) / 32;
+  if (kQ > 2 && nq <= 2) {
+    compact_selected(s_mask, a.N, s_list, s_wc);
+    refine_tokens_q<(kQ > 2 ? 2 : kQ)>(a, s_list, nS, t_begin, t_end, kp, row, ids_s);
+  } else if (kQ > 4 && nq <= 4) {
+    compact_selected(s_mask, a.N, s_list, s_wc);
+    refine_tokens_q<(kQ > 4 ? 4 : kQ)>(a, s_list, nS, t_begin, t_end, kp, row, ids_s);
+  } else {
+    refine_tokens_masked<kQ>(a, s_mask, t_begin, t_end, kp, row, ids_s);
   }
 }
 
@@ -821,7 +903,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   __syncthreads();
   int32_t *ids_s = C == 1 ? &s_top[0][0] : nullptr;  // one chunk: ids stay in shared memory
   refine_tokens<kQ>(
-      a, s_mask, 0, B, min(k, nsel),
+      a, s_mask, nsel, s_chunk, s_tmp, 0, B, min(k, nsel),
       [&](int t) -> const float * {
         // The chunk's rows hold the sparse values in that mode; refine on dense p.
         return (t >= t0 && t < t0 + nt && !a.sparse) ? ps + (t - t0) * N : a.p + (size_t)t * N;
@@ -852,7 +934,8 @@ __global__ void __launch_bounds__(kRouteThreads, 1) refine_kernel(RouteArgs a) {
   const int kp = a.meta->kprime;
   for (int j = tid; j < N; j += blockDim.x) s_mask[j] = a.mask[j];
   __syncthreads();
-  refine_tokens<kQ>(a, s_mask, t0, t0 + nt, kp, [&](int t) { return a.p + (size_t)t * N; });
+  refine_tokens<kQ>(a, s_mask, a.meta->n_selected, s_chunk, s_tmp, t0, t0 + nt, kp,
+                    [&](int t) { return a.p + (size_t)t * N; });
 
   // ---- the last CTA to finish builds the permutation (a7) ----
   __threadfence();
