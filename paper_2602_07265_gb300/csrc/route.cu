@@ -118,6 +118,51 @@ __device__ __forceinline__ int lane_take(LaneList<Q> &L, int count, Emit emit) {
   return r;
 }
 
+// Marks (calls mark(index) for) the `count` best candidates of an unsorted
+// lane list laid out by lane_load (lane l slot q: index j0 + l + 32 q), in
+// the order of `before`: every candidate whose key is above the count-th
+// largest key T, then the lowest-index candidates whose key equals T.  T is
+// found bit by bit from the top (the largest T with count(key >= T) >=
+// count), one warp reduction per bit.  All of them if count >= the live
+// candidates.
+template <int Q, class Mark>
+__device__ __forceinline__ void lane_mark_top(const LaneList<Q> &L, int count, Mark mark) {
+  const int lane = threadIdx.x & 31;
+  if (count <= 0) return;
+  int live = 0;
+#pragma unroll
+  for (int q = 0; q < Q; ++q) live += L.key[q] != 0u ? 1 : 0;
+  live = static_cast<int>(__reduce_add_sync(kFull, static_cast<unsigned>(live)));
+  if (count >= live) {
+#pragma unroll
+    for (int q = 0; q < Q; ++q)
+      if (L.key[q] != 0u) mark(L.idx[q]);
+    return;
+  }
+  uint32_t T = 0u;
+  for (int bit = 31; bit >= 0; --bit) {
+    const uint32_t c = T | (1u << bit);
+    int n = 0;
+#pragma unroll
+    for (int q = 0; q < Q; ++q) n += L.key[q] >= c ? 1 : 0;
+    if (static_cast<int>(__reduce_add_sync(kFull, static_cast<unsigned>(n))) >= count) T = c;
+  }
+  int gt = 0;
+#pragma unroll
+  for (int q = 0; q < Q; ++q) {
+    gt += L.key[q] > T ? 1 : 0;
+    if (L.key[q] > T) mark(L.idx[q]);
+  }
+  int need = count - static_cast<int>(__reduce_add_sync(kFull, static_cast<unsigned>(gt)));
+#pragma unroll
+  for (int q = 0; q < Q; ++q) {
+    const bool tie = L.key[q] == T;
+    const unsigned b = __ballot_sync(kFull, tie);
+    if (tie && __popc(b & ((1u << lane) - 1u)) < need) mark(L.idx[q]);
+    need -= __popc(b);
+  }
+}
+
 // Halving tree over the expert index of values held as v[q] = value of expert
 // lane + 32 q (zero where there is none): for o = 16 Q, ..., 32 the pairs
 // (j, j + o) are in one lane; for o = 16, ..., 1 they are lanes l and l + o.
@@ -871,10 +916,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
     LaneList<kQ> L;
     lane_load<kQ>(L, 0, N, lane, [&](int, int j) { return s_col[j]; },
                   [&](int, int j) { return s_base[j] == 0 && (!a.sparse || s_col[j] > 0.f); });
-    lane_sort<kQ>(L);
-    lane_take<kQ>(L, a.budget, [&](int, int id, float) {
-      if (lane == 0) s_mask[id] = 1;
-    });
+    lane_mark_top<kQ>(L, a.budget, [&](int id) { s_mask[id] = 1; });
   }
   __syncthreads();
 
