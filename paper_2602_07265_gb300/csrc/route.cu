@@ -254,20 +254,23 @@ __device__ __forceinline__ void block_scan3(int (&v)[3], int (&tot)[3], int *s_t
 // a single-pass evaluation):
 //
 //   score_kernel  (a2, a3, a4, part of a5): per token (one warp each) the
-//       dense softmax of the logits (or the given scores) and its ranked
-//       top-max(k, k0) over E; the chunk's column-sum tree; the chunk's
-//       warm-up and plain top-k union marks; for HIER, Algorithm 3 for every
-//       request inside the chunk.  The CTA that finishes last adds the chunk
-//       sums left to right, merges the marks and runs the budgeted selection
-//       (a5): BATCH and the batch step of HIER rank the column scores outside
-//       the base set in one warp; GROUP ranks each group in its own warp
-//       (Algorithm 5's rounds in closed form).
+//       dense softmax of the logits (or the given scores) and the ranking the
+//       selection needs (the warm-up top-k0; the top-k too for the sparse
+//       reading); the chunk's column-sum tree and warm-up marks; for HIER,
+//       Algorithm 3 for every request inside the chunk.  The CTA that
+//       finishes last adds the chunk sums left to right, merges the marks and
+//       runs the budgeted selection (a5): BATCH and the batch step of HIER
+//       search the budget-th column score outside the base set in one warp;
+//       GROUP ranks each group in its own warp (Algorithm 5's rounds in
+//       closed form).  CTAs C .. 2C - 1 rank every token's top-k over E at
+//       the same time and count the plain top-k union (a statistic).
 //   refine_kernel (a6, a7): per token the top-k' inside S with renormalised
 //       weights.  The CTA that finishes last counts the pairs per expert,
 //       takes the prefix sums, writes the FFN tiles and scatters the pairs
 //       stably by expert.
 //
-// "Last to finish" uses an arrival counter per kernel, cleared before the
+// "Last to finish" uses an arrival counter per group of CTAs (done[0] the
+// selection, done[1] the refinement, done[2] the union), cleared before the
 // first kernel of the call: every CTA writes its results, fences, and bumps
 // the counter; the CTA that sees the final count continues alone.  No CTA
 // waits for another.

@@ -114,7 +114,7 @@ struct RouteArgs {
   int32_t *perm_out;
   float *chunk_col;      // [C][N] column-sum tree of each 32-token chunk
   uint8_t *chunk_marks;  // [C][2][N] each chunk's warm-up / base marks and union marks
-  int32_t *done;         // [2] arrival counters of the two selection kernels, zero at entry
+  int32_t *done;         // [3] arrival counters (selection, refinement, union), zero at entry
   int32_t *zero_words;   // nullable: region cleared for the FFN kernels
   int zero_count;
   void *const *events;   // nullable: events[0] is recorded between the two kernels
