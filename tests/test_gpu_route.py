@@ -150,6 +150,39 @@ def test_route_edge_cases(X, B, N, k, budget, mode, params, ties):
     check(X, p, k, budget, mode, **params)
 
 
+def tied_boundary_scores(B, N, tied, high, seed):
+    """Scores whose column sums put a group of equal columns (`tied`, equal
+    entries in every row) right at the budget boundary, below the `high`
+    columns and above all the others; the per-token ranking ties too."""
+    rng = np.random.default_rng(seed)
+    p = (rng.uniform(0.5, 1.0, size=(B, N)) / (4.0 * N)).astype(np.float32)
+    p[:, high] = (rng.uniform(4.0, 8.0, size=(B, len(high))) / N).astype(np.float32)
+    p[:, tied] = np.float32(2.0 / N)
+    return p
+
+
+@pytest.mark.parametrize("k0,budget", [(0, 10), (0, 7), (1, 7), (0, 16)])
+def test_batch_ties_at_the_budget_boundary(X, k0, budget):
+    """BATCH takes the budget best columns in (score descending, index
+    ascending) order: with ten equal columns at the boundary the lowest
+    indices win, across the lanes and slots of the warp's candidate lists
+    (indices 3 .. 63 and, for N = 256, beyond 128)."""
+    for N, tied, high in ((64, [3, 17, 20, 33, 40, 41, 50, 58, 61, 63], [0, 9, 30, 31, 45, 60]),
+                          (256, [5, 37, 70, 99, 130, 131, 160, 200, 201, 255], [1, 2, 64, 128, 190, 254])):
+        p = tied_boundary_scores(32, N, tied, high, seed=N + budget)
+        ref = check(X, p, 8, budget, W.MODE_BATCH, k0=k0)
+        sel = set(np.flatnonzero(ref["mask"]).tolist())
+        assert set(high) <= sel or k0 > 0
+
+
+@pytest.mark.parametrize("B,N,budget,k0", [(32, 256, 24, 1), (64, 256, 40, 0), (96, 1024, 60, 2)])
+def test_refinement_over_a_short_selected_list_with_ties(X, B, N, budget, k0):
+    """Refinement over a compact list of S (|S| <= 128 with N >= 256):
+    per-token ties broken by the lower expert index, as over all N."""
+    p = W.random_scores(B, N, seed=B + N + budget, ties=True)
+    check(X, p, 8, budget, W.MODE_BATCH, k0=k0)
+
+
 def test_zero_rows_get_equal_weights(X):
     p = W.random_scores(12, 64, seed=3)
     p[[0, 5, 11]] = 0.0
