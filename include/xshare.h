@@ -25,6 +25,11 @@
  *     bounded wait that ran out) is reported in xs_stats.status, which the
  *     caller reads after synchronising.
  *   - Scores must be finite (no NaN): selection compares them as fp32 values.
+ *   - Host state: per-device caches of device properties (SM count, cluster
+ *     occupancy) and the driver's tensor-map encoder, filled on first use and
+ *     safe to fill from several host threads at once.  Calls on different
+ *     workspaces and streams may run concurrently (xshare_route_static
+ *     excepted, below).
  *
  * Limits: 1 <= N <= 1024 experts; 1 <= k <= min(N, 16); 0 <= k0 <= min(N, 16);
  * 1 <= B <= 8192 tokens; for the forward calls d % 128 == 0 and F % 128 == 0;
@@ -227,7 +232,7 @@ int xshare_moe_forward(const uint16_t *x, const float *W_g, const uint16_t *W_ga
  *     cudaGetSymbolAddress; make that first call before any stream capture;
  *   - every call on a device uses the same array, so calls that can overlap
  *     on the GPU (different streams, or different host threads) race and
- *     must be ordered by the caller.  Each call clears the two arrival
+ *     must be ordered by the caller.  Each call clears the three arrival
  *     counters it keeps in the array (a cudaMemsetAsync on `stream`); every
  *     other scratch word is written before it is read.
  * Allocates nothing (no cudaMalloc, cudaFree or allocating library call). */
@@ -238,8 +243,9 @@ int xshare_route_static(const float *scores, int B, int N, int k, int budget, in
 
 /* Kernel stages of xshare_moe_forward, in launch order: router logits,
  * selection (softmax, ranking, column scores, Algorithms 2-6), refinement
- * and permutation, token gather, SwiGLU gate/up, SwiGLU down, weighted
- * combine. */
+ * and permutation (inside the selection kernel for B <= 64, so its events
+ * then enclose no kernel), token gather, SwiGLU gate/up, SwiGLU down,
+ * weighted combine. */
 #define XS_N_STAGES 7
 
 /* xshare_moe_forward that also records CUDA events on `stream` between its

@@ -2,6 +2,7 @@
 // and the stream-ordered launch sequence of the MoE-layer forward.
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cstdint>
 #include <cstring>
 
@@ -14,29 +15,26 @@ constexpr size_t kAlign = 256;
 
 size_t align_up(size_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
 
-struct DevInfo {
-  int known;
-  int ok;
-  int n_sms;
-};
-DevInfo g_dev[64];
+// Per device: 0 until known, then the SM count of an sm_103 device or
+// XS_ERR_DEVICE.  Filled on first use; host threads that race on it store
+// the same value.
+std::atomic<int> g_dev_sms[64];
 
 // The current device's SM count, or a negative XS_ERR code.
 int current_device_sms() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return XS_ERR_CUDA;
-  DevInfo &di = g_dev[dev];
-  if (!di.known) {
+  int v = g_dev_sms[dev].load(std::memory_order_relaxed);
+  if (v == 0) {
     int major = 0, minor = 0, sms = 0;
     if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
       return XS_ERR_CUDA;
-    di.ok = (major == 10 && minor == 3);
-    di.n_sms = sms;
-    di.known = 1;
+    v = (major == 10 && minor == 3 && sms > 0) ? sms : XS_ERR_DEVICE;
+    g_dev_sms[dev].store(v, std::memory_order_relaxed);
   }
-  return di.ok ? di.n_sms : XS_ERR_DEVICE;
+  return v;
 }
 
 int check_route_args(int B, int N, int k, int budget, int mode, const xs_route_params *prm) {

@@ -35,6 +35,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cstring>
 
 #include "tc_ptx.cuh"
@@ -316,39 +317,38 @@ KernelFn kernel_for(int nt) {
 }
 
 // Clusters of S CTAs of the nt variant that the current device can hold at
-// once (cached per device); 0 if the query fails.
+// once (cached per device; host threads that race on it store the same
+// value); 0 if the query fails.
 int cluster_cap(int nt, int S) {
   constexpr int kDevs = 64;
-  static int cache[kDevs][3][5];
-  static bool known[kDevs][3][5];
+  static std::atomic<int> cache[kDevs][3][5];  // the count + 1, 0 while unknown
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kDevs) return 0;
   const int a = nt == 16 ? 0 : nt == 32 ? 1 : 2;
   const int b = S == 1 ? 0 : S == 2 ? 1 : S == 4 ? 2 : S == 8 ? 3 : 4;
-  if (!known[dev][a][b]) {
-    int n = 0;
-    const KernelFn k = kernel_for(nt);
-    if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(smem_for(nt))) == cudaSuccess &&
-        cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
-      cudaLaunchConfig_t cfg = {};
-      cfg.gridDim = dim3(S);
-      cfg.blockDim = dim3(kThreads);
-      cfg.dynamicSmemBytes = smem_for(nt);
-      cudaLaunchAttribute attr[1];
-      attr[0].id = cudaLaunchAttributeClusterDimension;
-      attr[0].val.clusterDim.x = S;
-      attr[0].val.clusterDim.y = 1;
-      attr[0].val.clusterDim.z = 1;
-      cfg.attrs = attr;
-      cfg.numAttrs = 1;
-      if (cudaOccupancyMaxActiveClusters(&n, k, &cfg) != cudaSuccess) n = 0;
-    }
-    cudaGetLastError();  // a failed query leaves no sticky error
-    cache[dev][a][b] = n;
-    known[dev][a][b] = true;
+  const int known = cache[dev][a][b].load(std::memory_order_relaxed);
+  if (known > 0) return known - 1;
+  int n = 0;
+  const KernelFn k = kernel_for(nt);
+  if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(smem_for(nt))) == cudaSuccess &&
+      cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(S);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem_for(nt);
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = S;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaOccupancyMaxActiveClusters(&n, k, &cfg) != cudaSuccess) n = 0;
   }
-  return cache[dev][a][b];
+  cudaGetLastError();  // a failed query leaves no sticky error
+  cache[dev][a][b].store(n + 1, std::memory_order_relaxed);
+  return n;
 }
 
 // Experts per tile (nt) and CTAs per cluster (S).  A CTA's time is a fixed
