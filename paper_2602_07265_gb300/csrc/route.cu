@@ -123,8 +123,9 @@ __device__ __forceinline__ int lane_take(LaneList<Q> &L, int count, Emit emit) {
 // the order of `before`: every candidate whose key is above the count-th
 // largest key T, then the lowest-index candidates whose key equals T.  T is
 // found bit by bit from the top (the largest T with count(key >= T) >=
-// count), one warp reduction per bit.  All of them if count >= the live
-// candidates.
+// count), one warp reduction per bit; the search stops early once a
+// threshold has exactly `count` keys at or above it.  All of them if count
+// >= the live candidates.
 template <int Q, class Mark>
 __device__ __forceinline__ void lane_mark_top(const LaneList<Q> &L, int count, Mark mark) {
   const int lane = threadIdx.x & 31;
@@ -145,7 +146,16 @@ __device__ __forceinline__ void lane_mark_top(const LaneList<Q> &L, int count, M
     int n = 0;
 #pragma unroll
     for (int q = 0; q < Q; ++q) n += L.key[q] >= c ? 1 : 0;
-    if (static_cast<int>(__reduce_add_sync(kFull, static_cast<unsigned>(n))) >= count) T = c;
+    n = static_cast<int>(__reduce_add_sync(kFull, static_cast<unsigned>(n)));
+    if (n == count) {
+      // Exactly `count` keys are >= c and every other key is below c: they
+      // are the count best, whatever the order among them.
+#pragma unroll
+      for (int q = 0; q < Q; ++q)
+        if (L.key[q] >= c) mark(L.idx[q]);
+      return;
+    }
+    if (n > count) T = c;
   }
   int gt = 0;
 #pragma unroll
