@@ -1131,24 +1131,41 @@ __global__ void __launch_bounds__(256) combine_kernel(const float *__restrict__ 
                                                       const uint16_t *__restrict__ resid,
                                                       uint16_t *__restrict__ y, int B, int d,
                                                       int k, int n_shared) {
-  pdl_wait();
-  pdl_trigger();
+  __shared__ int32_t s_row[kMaxK];
+  __shared__ float s_w[kMaxK];
+  __shared__ int32_t s_kp, s_pairs;
   const int t = blockIdx.y;
   const int c4 = blockIdx.x * blockDim.x + threadIdx.x;
-  if (c4 >= d / 4) return;
-  const int kp = meta->kprime;
+  // Before pdl_wait(): the token's rows and weights and the pair count,
+  // written by the routing kernels four launches earlier (complete before
+  // this grid started), and x_t (an input, or the previous layer's output);
+  // only `out` comes from the kernel just before.
+  if (threadIdx.x < kMaxK) {
+    const int s = threadIdx.x;
+    s_row[s] = s < k ? __ldcg(pos + (size_t)t * k + s) : -1;
+    s_w[s] = s < k ? __ldcg(w + (size_t)t * k + s) : 0.f;
+  }
+  if (threadIdx.x == 0) {
+    s_kp = __ldcg(&meta->kprime);
+    s_pairs = __ldcg(&meta->n_pairs);
+  }
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  if (resid != nullptr) {
-    const uint2 r = reinterpret_cast<const uint2 *>(resid + (size_t)t * d)[c4];
+  if (resid != nullptr && c4 < d / 4) {
+    const uint2 r = __ldcg(reinterpret_cast<const uint2 *>(resid + (size_t)t * d) + c4);
     acc.x = __uint_as_float(r.x << 16);
     acc.y = __uint_as_float(r.x & 0xffff0000u);
     acc.z = __uint_as_float(r.y << 16);
     acc.w = __uint_as_float(r.y & 0xffff0000u);
   }
+  __syncthreads();
+  pdl_wait();
+  pdl_trigger();
+  if (c4 >= d / 4) return;
+  const int kp = s_kp;
   for (int s = 0; s < kp; ++s) {
-    const int r = pos[(size_t)t * k + s];
+    const int r = s_row[s];
     if (r < 0) continue;  // only with non-finite scores
-    const float ws = w[(size_t)t * k + s];
+    const float ws = s_w[s];
     const float4 o = reinterpret_cast<const float4 *>(out + (size_t)r * d)[c4];
     acc.x = fmaf(ws, o.x, acc.x);
     acc.y = fmaf(ws, o.y, acc.y);
@@ -1156,7 +1173,7 @@ __global__ void __launch_bounds__(256) combine_kernel(const float *__restrict__ 
     acc.w = fmaf(ws, o.w, acc.w);
   }
   for (int j = 0; j < n_shared; ++j) {
-    const size_t r = (size_t)meta->n_pairs + (size_t)j * B + t;
+    const size_t r = (size_t)s_pairs + (size_t)j * B + t;
     const float4 o = reinterpret_cast<const float4 *>(out + r * d)[c4];
     acc.x += o.x;
     acc.y += o.y;

@@ -18,8 +18,9 @@ namespace xs {
 // CTA waits before it exits.  Hence when a CTA of kernel n starts, kernel
 // n - 2 and everything before it have completed: the FFN kernels read the
 // routing results (written two or more launches earlier) and start their
-// weight loads before pdl_wait(); every other access to global memory, in
-// every kernel, comes after it.
+// weight loads before pdl_wait(), and the combine kernel reads its rows,
+// weights and x_t then; every other access to global memory, in every
+// kernel, comes after it.
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
