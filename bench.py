@@ -1,5 +1,5 @@
 #!/usr/bin/env python
-"""Benchmark of one XShare MoE-layer forward on GB300 (see the design doc for the recipe).
+"""Benchmark of one XShare MoE-layer forward on GB300.
 
 A step is one xshare_moe_forward call: router + softmax, batch-aware expert
 selection, refinement, permutation, gather, SwiGLU expert FFN over the used
@@ -46,6 +46,7 @@ METRIC = "MoE-layer tokens/s and expert-weight HBM GB/s (% roofline); experts ac
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 N_ROTATE = 4   # distinct input batches cycled through the timed steps
+L2_BYTES = 129e6
 
 
 # --------------------------------------------------------------------------- setup
@@ -128,6 +129,22 @@ def describe(w: W.Workload, n_shared: int = 0) -> str:
     if n_shared:
         s += f" + {n_shared} shared expert{'s' if n_shared > 1 else ''}"
     return s
+
+
+def workload_config(w: W.Workload, n_shared: int, world: int) -> dict:
+    """The `config` of the JSON line, the same for both arms: the workload and
+    how the timed steps stay clear of L2."""
+    return {
+        "workload": describe(w, n_shared),
+        "B": w.B, "N": w.N, "k": w.k, "d": w.d, "F": w.F, "shared_experts": n_shared,
+        "global_batch": w.B * world,
+        "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+        "l2": (f"inputs larger than L2: every step streams the weights of its used experts "
+               f"({w.expert_bytes / 1e6:.1f} MB each; L2 129 MB), {N_ROTATE} rotating input batches")
+        if w.N * w.expert_bytes > L2_BYTES else
+        (f"all expert weights fit in L2 ({w.N * w.expert_bytes / 1e6:.0f} MB of 129 MB): "
+         f"L2-warm steps, a correctness-size workload, not a bandwidth figure"),
+    }
 
 
 def measured_peaks() -> dict:
@@ -457,16 +474,10 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic",
-        "config": {
-            "workload": describe(w, Ns),
-            "B": w.B, "N": w.N, "k": w.k, "d": w.d, "F": w.F, "shared_experts": Ns,
-            "expert_weights": "packed 128 x 64 tiles (xshare_pack_experts, once at load)"
-                              if packed else "plain [N, F, d] / [N, d, F] matrices",
-            "global_batch": w.B * world,
-            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-            "l2": f"inputs larger than L2: ~{layer_bytes / 1e9:.2f} GB of expert weights per step "
-                  f"(L2 129 MB), {N_ROTATE} rotating input batches",
-        },
+        "config": workload_config(w, Ns, world),
+        "expert_weights": "packed 128 x 64 tiles (xshare_pack_experts, once at load)"
+                          if packed else "plain [N, F, d] / [N, d, F] matrices",
+        "weights_streamed_gb_per_step": layer_bytes / 1e9,
         "experts": {
             "selected_mean": float(st[:, 0].mean()), "used_mean": float(n_used.mean()),
             "union_topk_mean": float(st[:, 2].mean()), "max_group_load_mean": float(st[:, 3].mean()),
@@ -630,112 +641,99 @@ def run_gpu_stack(args, w: W.Workload, rank: int, world: int, local: int) -> dic
 
 # --------------------------------------------------------------------------- oracle timing
 
-class OracleSampler:
-    """Times the CPU oracle on a bounded sample of one step of workload `w`:
-    the full selection for the batch (router, softmax, Algorithms 2-6,
-    refinement, permutation), plus the expert FFN and combine of `ffn_tokens`
-    tokens restricted to the first `f_rows` hidden units of each expert.  The
-    SwiGLU output is a sum over hidden units, so the FFN time is scaled by
-    F / f_rows.  Inputs and the needed expert weights are prepared once,
-    outside the timed calls."""
+class OracleStep:
+    """One whole layer step of the CPU oracle on workload `w`: router logits,
+    softmax, selection (Algorithms 2-6), refinement, permutation, the expert
+    FFN of every routed (token, slot) pair on all F hidden units, the shared
+    experts and the weighted combine, for all B tokens of one input batch, in
+    fp64 with numpy.  The inputs and the bf16 weights of the experts this
+    batch uses are drawn once, outside the timed calls; the oracle widens them
+    to fp64 inside every step, as it stands."""
 
-    def __init__(self, w: W.Workload, seed: int, ffn_tokens: int, f_rows: int,
-                 n_shared: int = 0):
+    def __init__(self, w: W.Workload, seed: int, n_shared: int = 0):
         from oracle import xshare_oracle as O
         self.O, self.w, self.n_shared = O, w, n_shared
-        self.f_rows = min(f_rows, w.F)
         x, W_g = W.router_inputs(w, seed)
         self.xb, self.W_g = W.bf16_bits(x), W_g.numpy()
         p = O.softmax_scores(O.router_logits(self.xb, self.W_g))
         r = O.route(p, w.k, w.budget, w.mode, **w.params())
-        self.tokens = list(range(min(ffn_tokens, w.B)))
-        self.experts = sorted({int(e) for t in self.tokens for e in r["ids"][t] if e >= 0})
+        self.experts = sorted(int(e) for e in r["used"])
         self.weights = {}
         if self.experts:
-            Wg, Wu, Wd = W.expert_weights(w, seed, device="cpu", experts=self.experts,
-                                          f_rows=self.f_rows)
+            Wg, Wu, Wd = W.expert_weights(w, seed, device="cpu", experts=self.experts)
             for i, e in enumerate(self.experts):
                 self.weights[e] = (W.bf16_bits(Wg[i]), W.bf16_bits(Wu[i]), W.bf16_bits(Wd[i]))
+            del Wg, Wu, Wd
         self.shared = []
         if n_shared:
-            Sg, Su, Sd = W.expert_weights(w.with_(N=n_shared), seed + 7_777_777, device="cpu",
-                                          f_rows=self.f_rows)
+            Sg, Su, Sd = W.shared_expert_weights(w, n_shared, seed, device="cpu")
             self.shared = [(W.bf16_bits(Sg[j]), W.bf16_bits(Su[j]), W.bf16_bits(Sd[j]))
                            for j in range(n_shared)]
 
-    def step(self) -> dict:
+    def step(self) -> float:
+        """Runs one step; returns its wall-clock seconds."""
         O, w = self.O, self.w
         t0 = time.perf_counter()
-        h = O.router_logits(self.xb, self.W_g)
-        p = O.softmax_scores(h)
-        r = O.route(p, w.k, w.budget, w.mode, **w.params())
-        t_route = time.perf_counter() - t0
-        t1 = time.perf_counter()
-        if self.tokens:
-            O.moe_ffn_combine(self.xb, r["ids"], r["w"], self.weights.__getitem__, tokens=self.tokens)
-            if self.n_shared:
-                O.shared_experts_out(self.xb, self.shared.__getitem__, self.n_shared, self.tokens)
-        t_ffn = (time.perf_counter() - t1) * (w.F / self.f_rows)
-        per_token = t_route / w.B + (t_ffn / len(self.tokens) if self.tokens else 0.0)
-        return {"t_route": t_route, "t_ffn_scaled": t_ffn, "per_token_s": per_token}
+        r = O.moe_forward(self.xb, self.W_g, self.weights.__getitem__, w.k, w.budget, w.mode,
+                          get_shared=self.shared.__getitem__ if self.n_shared else None,
+                          n_shared=self.n_shared, **w.params())
+        dt = time.perf_counter() - t0
+        assert r["y"].shape == (w.B, w.d)
+        return dt
 
-    def describe(self, s: dict) -> str:
-        sh = f" (+ {self.n_shared} shared)" if self.n_shared else ""
-        return (f"full selection of one {self.w.B}-token batch ({s['t_route']:.2f} s) + expert FFN{sh} "
-                f"and combine of {len(self.tokens)} token(s) on {self.f_rows}/{self.w.F} hidden units, "
-                f"scaled to F ({s['t_ffn_scaled']:.2f} s); numpy fp64, 1 thread")
+    def describe(self) -> str:
+        sh = f" and {self.n_shared} shared" if self.n_shared else ""
+        return (f"full layer steps on one {self.w.B}-token batch: router, softmax, selection, "
+                f"refinement, permutation, SwiGLU FFN of all {self.w.B} tokens over its "
+                f"{len(self.experts)} used experts{sh} on all {self.w.F} hidden units, combine; "
+                f"numpy fp64, 1 thread")
 
 
-def cpu_baseline(w: W.Workload, seed: int, n_shared: int = 0) -> dict:
-    """The oracle, single-threaded, on a bounded sample, in a child process so
-    that BLAS is pinned to one thread."""
+def cpu_baseline(w: W.Workload, seed: int, n_shared: int = 0, steps: int = 2) -> dict:
+    """The oracle, single-threaded, timed over `steps` whole layer steps after
+    one untimed step, in a child process so that BLAS is pinned to one thread."""
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
                CUDA_VISIBLE_DEVICES="")
-    f_rows = max(128, w.F // 4)
     kw = json.dumps(dict(B=w.B, N=w.N, F=w.F, budget=w.budget, k0=w.k0, mode=w.mode, tau=w.tau,
                          sparse_scores=w.sparse_scores, m_r=w.m_r, m_g=w.m_g))
     code = (f"import sys, json; sys.path.insert(0, {ROOT!r}); import torch; torch.set_num_threads(1); "
             f"import bench; from paper_2602_07265_gb300 import workloads as W; "
             f"w = W.WORKLOADS[{w.name!r}].with_(**{kw}); "
-            f"o = bench.OracleSampler(w, {seed}, 4, {f_rows}, {int(n_shared)}); o.step(); s = o.step(); "
-            f"s['describe'] = o.describe(s); print(json.dumps(s))")
+            f"o = bench.OracleStep(w, {seed}, {int(n_shared)}); o.step(); "
+            f"t = [o.step() for _ in range({int(steps)})]; "
+            f"print(json.dumps(dict(t=t, describe=o.describe())))")
     r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
-                       timeout=900)
+                       timeout=1800)
     if r.returncode != 0:
         tail = r.stderr.strip().splitlines()[-1][:200] if r.stderr.strip() else "no output"
         return {"value": None, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                 "sample": "failed: " + tail}
     s = json.loads(r.stdout.strip().splitlines()[-1])
-    return {"value": 1.0 / s["per_token_s"], "unit": "tokens/s", "cores": 1, "kind": "oracle",
-            "sample": s["describe"]}
+    mean_s = float(np.mean(s["t"]))
+    return {"value": w.B / mean_s, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+            "sample": f"{len(s['t'])} timed {s['describe']} (mean {mean_s:.2f} s per step)"}
 
 
 def run_reference(args, w: W.Workload, rank: int, world: int) -> dict:
-    """The oracle as the reference arm: K timed steps, each a bounded sample
-    of one step of the same workload, single-threaded on the host cores.
-    Steps beyond a ~150 s budget are skipped, keeping at least 3."""
+    """The oracle as the reference arm: W untimed and K timed whole layer steps
+    of the same workload (one input batch), single-threaded on the host
+    cores; ms_per_step is the measured mean of the K steps."""
     torch.set_num_threads(1)
     K, Wm = args.steps, args.warmup
-    sampler = OracleSampler(w, args.seed, 1, max(128, w.F // 8), args.shared)
-    for _ in range(min(Wm, 3)):
-        s = sampler.step()
-    budget_s, spent, per_token = 150.0, 0.0, []
-    for i in range(K):
-        t = time.perf_counter()
-        s = sampler.step()
-        spent += time.perf_counter() - t
-        per_token.append(s["per_token_s"])
-        if spent > budget_s and i >= 2:
-            break
-    value = 1.0 / float(np.mean(per_token))
-    sample = f"{len(per_token)} of {K} steps timed; each: " + sampler.describe(s)
+    oracle = OracleStep(w, args.seed, args.shared)
+    for _ in range(Wm):
+        oracle.step()
+    times = [oracle.step() for _ in range(K)]
+    mean_s = float(np.mean(times))
+    value = w.B / mean_s
+    sample = f"{K} timed {oracle.describe()} (median {1e3 * float(np.median(times)):.0f} ms)"
     return {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
-        "warmup": Wm, "ms_per_step": 1e3 * w.B / value, "higher_is_better": True,
+        "warmup": Wm, "ms_per_step": 1e3 * mean_s, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "impl": "reference",
-        "config": {"workload": describe(w, args.shared), "B": w.B, "N": w.N, "k": w.k, "d": w.d,
-                   "F": w.F, "shared_experts": args.shared, "global_batch": w.B, "parallelism": "cpu oracle, rank 0 only"},
+        "config": workload_config(w, args.shared, world),
+        "runs_on": "host cores, rank 0 only",
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,

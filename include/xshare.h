@@ -229,7 +229,10 @@ int xshare_moe_forward(const uint16_t *x, const float *W_g, const uint16_t *W_ga
  *     larger B returns XS_ERR_SHAPE and launches nothing;
  *   - only the dense scores: prm->sparse_scores != 0 returns XS_ERR_PARAM;
  *   - the first call on a device looks up the array's device address with
- *     cudaGetSymbolAddress; make that first call before any stream capture;
+ *     cudaGetSymbolAddress; make that first call before any stream capture.
+ *     The address belongs to the device's current CUDA context: after a
+ *     cudaDeviceReset (or any new context on the device) the next call looks
+ *     it up again, so that call, too, must come before any stream capture;
  *   - every call on a device uses the same array, so calls that can overlap
  *     on the GPU (different streams, or different host threads) race and
  *     must be ordered by the caller.  Each call clears the three arrival

@@ -8,9 +8,12 @@
 // keeps its scratch in a fixed array that the library module itself defines
 // in device memory, sized for at most kStaticMaxB tokens, so the caller passes
 // only its inputs and outputs.
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 #include <cstring>
+#include <mutex>
 
 #include "xs_internal.cuh"
 
@@ -45,7 +48,64 @@ constexpr size_t kStaticBytes = kOffDone + up256(4 * sizeof(int32_t));
 static __device__ __align__(256) unsigned char g_route_scratch[kStaticBytes];
 
 constexpr int kMaxDevices = 64;
-void *g_scratch_addr[kMaxDevices];  // device address of g_route_scratch, per device
+
+// Where g_route_scratch lives on a device, valid for one CUDA context of that
+// device: a cudaDeviceReset destroys the primary context and with it the
+// module's copy of the array, and the next context loads a new copy at
+// another address.  The address is therefore kept with the unique id of the
+// context it was looked up in and looked up again when the current context
+// has another id.  The mutex makes the set-up safe when host threads race
+// on it.
+struct ScratchAddr {
+  std::mutex mu;
+  unsigned long long ctx_id = 0;
+  bool valid = false;
+  void *addr = nullptr;
+};
+ScratchAddr g_scratch[kMaxDevices];
+
+// The driver's cuCtxGetCurrent and cuCtxGetId, through the runtime's entry
+// point query (the library does not link libcuda).  Function-local statics
+// are initialised once even when threads race on the first call.
+template <class Fn>
+Fn driver_fn(const char *name, int version) {
+  void *ptr = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion(name, &ptr, version, cudaEnableDefault, &q) == cudaSuccess &&
+      q == cudaDriverEntryPointSuccess)
+    return reinterpret_cast<Fn>(ptr);
+  return nullptr;
+}
+
+// Id of the context current on this thread; false if there is none.
+bool current_context_id(unsigned long long *id) {
+  static const PFN_cuCtxGetCurrent_v4000 get_current =
+      driver_fn<PFN_cuCtxGetCurrent_v4000>("cuCtxGetCurrent", 4000);
+  static const PFN_cuCtxGetId_v12000 get_id = driver_fn<PFN_cuCtxGetId_v12000>("cuCtxGetId", 12000);
+  if (get_current == nullptr || get_id == nullptr) return false;
+  CUcontext ctx = nullptr;
+  if (get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return false;
+  return get_id(ctx, id) == CUDA_SUCCESS;
+}
+
+// Device address of g_route_scratch in the current context of device `dev`
+// (the current device), or nullptr on a CUDA error.  The look-up runs on the
+// first call in each context of the device; later calls reuse it.
+void *scratch_address(int dev) {
+  ScratchAddr &slot = g_scratch[dev];
+  std::lock_guard<std::mutex> lock(slot.mu);
+  unsigned long long id = 0;
+  if (slot.valid && current_context_id(&id) && id == slot.ctx_id) return slot.addr;
+  // Set-up: cudaGetSymbolAddress also makes the device's primary context
+  // current if no context was yet.
+  void *addr = nullptr;
+  if (cudaGetSymbolAddress(&addr, g_route_scratch) != cudaSuccess || addr == nullptr) return nullptr;
+  if (!current_context_id(&id)) return nullptr;
+  slot.addr = addr;
+  slot.ctx_id = id;
+  slot.valid = true;
+  return addr;
+}
 
 }  // namespace
 }  // namespace xs
@@ -81,14 +141,8 @@ extern "C" int xshare_route_static(const float *scores, int B, int N, int k, int
       cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
     return XS_ERR_CUDA;
   if (major != 10 || minor != 3) return XS_ERR_DEVICE;
-  if (g_scratch_addr[dev] == nullptr) {
-    // One-time set-up on this device: look up where the scratch array lives.
-    void *addr = nullptr;
-    if (cudaGetSymbolAddress(&addr, g_route_scratch) != cudaSuccess || addr == nullptr)
-      return XS_ERR_CUDA;
-    g_scratch_addr[dev] = addr;
-  }
-  char *base = static_cast<char *>(g_scratch_addr[dev]);
+  char *base = static_cast<char *>(scratch_address(dev));
+  if (base == nullptr) return XS_ERR_CUDA;
 
   RouteArgs a;
   std::memset(&a, 0, sizeof(a));

@@ -12,7 +12,10 @@ Checks:
   tolerance (checked, never assumed);
 * output: max|y - y_ref| / max|y_ref| <= 2e-2 and ||y - y_ref||_F / ||y_ref||_F
   <= 1e-2 (bf16 output of an fp32-accumulated path with a bf16 activation).
-At the full DeepSeek-R1 shapes the oracle evaluates sampled tokens only.
+At the DeepSeek-R1 shapes up to B = 128 every token is compared; at B = 256
+the first 128 tokens (one full 128-row FFN tile's worth).  Each comparison
+records whether the near-tie rule (below) had to drop tokens; a last test in
+this file bounds how often that happened.
 """
 import numpy as np
 import pytest
@@ -100,6 +103,13 @@ def robust_selection(p, w: W.Workload, rtol: float, trials: int = 6) -> bool:
     return True
 
 
+# One entry per compare() call: (case label, tokens dropped by the near-tie rule).
+NEAR_TIE_LOG = []
+# At most this fraction of the compared cases may fall back to the near-tie
+# rule (routing differing from the oracle's on a near-tie of its fp32 scores).
+NEAR_TIE_MAX_FRACTION = 0.05
+
+
 def compare(w, g, x, W_g, weights, tokens=None, shared=None):
     """Check a GPU forward against the oracle; returns (ref, max_rel, fro, n_tokens_compared).
 
@@ -131,8 +141,11 @@ def compare(w, g, x, W_g, weights, tokens=None, shared=None):
         assert not robust_selection(ref["p"], w, eps), \
             "routing differs from the oracle's although its decision is not near a tie"
     keep = [i for i, t in enumerate(toks) if same_row[t]]
+    dropped = len(toks) - len(keep)
+    NEAR_TIE_LOG.append((f"{w.name} B={w.B} mode={w.mode}", dropped, same_mask))
     print(f"[{w.name} B={w.B} mode={w.mode}] p_rel_max={rel.max():.2e} same_mask={same_mask} "
-          f"same_rows={int(same_row.sum())}/{w.B} compared={len(keep)}/{len(toks)}")
+          f"same_rows={int(same_row.sum())}/{w.B} compared={len(keep)}/{len(toks)}"
+          + (f" NEAR-TIE FALLBACK: {dropped} token(s) dropped" if dropped or not same_mask else ""))
     assert len(keep) >= max(1, (3 * len(toks)) // 4), "too few tokens with identical routing"
     rows = [toks[i] for i in keep]
     assert np.allclose(g["w"][rows], ref["w"][rows], rtol=4 * P_RTOL, atol=0), "weights"
@@ -176,18 +189,68 @@ def test_forward_parity_small(X, case, seed):
     compare(w, g, x, W_g, weights)
 
 
-@pytest.mark.parametrize("w", [
+FULL_SIZE = [
     W.DSR1.with_(B=8), W.DSR1, W.DSR1.with_(B=128, budget=64), W.DSR1.with_(k0=0, budget=32),
     W.DSR1_GROUP, W.DSR1_GROUP.with_(k0=0, m_g=8), W.DSR1.with_(mode=W.MODE_THRESH, tau=0.5),
     W.DSR1.with_(budget=40, sparse_scores=1),
-], ids=lambda w: f"{w.name}-B{w.B}-m{w.budget}-k0{w.k0}-mg{w.m_g}-mode{w.mode}-s{w.sparse_scores}")
-def test_forward_parity_full_size_sampled(X, w):
-    """DeepSeek-R1-shaped layers at full size; the oracle checks sampled tokens."""
+]
+
+
+def full_size_tokens(w):
+    """Every token up to B = 128; beyond, the first 128 (a full FFN tile's rows)."""
+    return None if w.B <= 128 else list(range(128))
+
+
+@pytest.mark.parametrize("w", FULL_SIZE,
+                         ids=lambda w: f"{w.name}-B{w.B}-m{w.budget}-k0{w.k0}-mg{w.m_g}-mode{w.mode}"
+                                       f"-s{w.sparse_scores}")
+def test_forward_parity_full_size(X, w):
+    """DeepSeek-R1-shaped layers at full size (d = 7168, F = 2048: 112 K-steps of
+    64 in gate/up, 32 in down, split across CTAs by the stream-K schedule),
+    compared with the oracle token by token."""
     x, W_g = W.router_inputs(w, 0)
     weights = device_weights(w, 0)
     g = gpu_forward(X, w, x, W_g, weights)
-    tokens = sorted({0, 1, w.B // 2, w.B - 1})
-    compare(w, g, x, W_g, weights, tokens=tokens)
+    compare(w, g, x, W_g, weights, tokens=full_size_tokens(w))
+
+
+def gpu_forward_packed(X, w: W.Workload, x, W_g, weights):
+    """xshare_moe_forward_packed (the path bench.py times) with the same outputs
+    as gpu_forward."""
+    dev = torch.device("cuda")
+    pk = X.Packed(*weights)
+    prm = X.route_params(**w.params())
+    ws = torch.empty(X.xshare_workspace_size(w.B, w.N, w.k, w.d, w.F, w.mode, prm, 0),
+                     dtype=torch.uint8, device=dev)
+    out = dict(
+        y=torch.empty(w.B, w.d, dtype=torch.bfloat16, device=dev),
+        p=torch.empty(w.B, w.N, dtype=torch.float32, device=dev),
+        mask=torch.empty(w.N, dtype=torch.uint8, device=dev),
+        ids=torch.empty(w.B, w.k, dtype=torch.int32, device=dev),
+        w=torch.empty(w.B, w.k, dtype=torch.float32, device=dev),
+        stats=torch.zeros(8, dtype=torch.int32, device=dev),
+    )
+    X.xshare_moe_forward_packed(x.to(dev), W_g.to(dev), pk, w.k, w.budget, w.mode, prm,
+                                out["y"], ws, scores_out=out["p"], sel_mask=out["mask"],
+                                topk_ids=out["ids"], topk_w=out["w"], stats=out["stats"])
+    torch.cuda.synchronize()
+    del pk
+    r = {name: t.cpu() for name, t in out.items()}
+    r["stats"] = X.stats_dict(out["stats"])
+    r["y"] = r["y"].float().numpy().astype(np.float64)
+    for name in ("p", "mask", "ids", "w"):
+        r[name] = r[name].numpy()
+    return r
+
+
+@pytest.mark.parametrize("w", [W.DSR1, W.DSR1.with_(B=8)], ids=lambda w: f"{w.name}-B{w.B}")
+def test_forward_packed_parity_full_size(X, w):
+    """The benchmarked path itself, xshare_moe_forward_packed on packed expert
+    weights at the DeepSeek-R1 shape, against the oracle on every token."""
+    x, W_g = W.router_inputs(w, 1)
+    weights = device_weights(w, 1)
+    g = gpu_forward_packed(X, w, x, W_g, weights)
+    compare(w, g, x, W_g, weights)
 
 
 @pytest.mark.parametrize("budget,k0", [(0, 0), (3, 0), (0, 1)])
@@ -311,3 +374,14 @@ def test_forward_limits(X, w, tokens):
     weights = device_weights(w, 7)
     g = gpu_forward(X, w, x, W_g, weights)
     compare(w, g, x, W_g, weights, tokens=tokens)
+
+
+def test_zz_near_tie_fallback_rate():
+    """The near-tie rule of compare() is a rare exception, not a way around
+    the comparison: it may fire on at most NEAR_TIE_MAX_FRACTION of the cases
+    this file compared (run after them: pytest keeps the file order)."""
+    if len(NEAR_TIE_LOG) < 20:
+        pytest.skip("needs the other forward parity tests of this file in the same run")
+    fired = [(c, n) for c, n, same_mask in NEAR_TIE_LOG if n or not same_mask]
+    print(f"near-tie fallback fired on {len(fired)} of {len(NEAR_TIE_LOG)} compared cases: {fired}")
+    assert len(fired) <= NEAR_TIE_MAX_FRACTION * len(NEAR_TIE_LOG), fired

@@ -11,6 +11,7 @@ import os
 import socket
 import subprocess
 import sys
+import time
 
 import pytest
 import torch.multiprocessing as mp
@@ -67,9 +68,11 @@ def test_single_rank_reductions_are_identity():
 def test_reference_arm_runs_on_rank_zero_only(rank):
     env = dict(os.environ, RANK=str(rank), WORLD_SIZE="2", LOCAL_RANK=str(rank),
                MASTER_ADDR="127.0.0.1", MASTER_PORT=str(_free_port()))
+    t0 = time.perf_counter()
     r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
                         "--workload", "tiny", "--steps", "3", "--warmup", "3"],
                        env=env, capture_output=True, text=True, timeout=300, cwd=ROOT)
+    wall_s = time.perf_counter() - t0
     assert r.returncode == 0, r.stderr
     lines = [l for l in r.stdout.splitlines() if l.strip()]
     if rank == 0:
@@ -77,5 +80,15 @@ def test_reference_arm_runs_on_rank_zero_only(rank):
         assert d["impl"] == "reference" and d["value"] > 0 and d["n_gpus"] == 2
         assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] == 1
         assert d["e2e"]["h2d_bytes_per_step"] == 0
+        # Whole layer steps, measured: the K timed steps fit inside the run, and
+        # the rate is the batch over the measured mean step time.
+        assert "full layer steps" in d["cpu_baseline"]["sample"]
+        assert d["steps"] == 3 and d["ms_per_step"] * d["steps"] * 1e-3 < wall_s
+        assert abs(d["value"] - 32 / (d["ms_per_step"] * 1e-3)) < 1e-6 * d["value"]
+        # The same config object as the GPU arm's line.
+        sys.path.insert(0, ROOT)
+        import bench
+        from paper_2602_07265_gb300 import workloads as W
+        assert d["config"] == json.loads(json.dumps(bench.workload_config(W.TINY, 0, 2)))
     else:
         assert lines == []

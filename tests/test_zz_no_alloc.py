@@ -6,16 +6,20 @@ a serving loop that must not call cudaMalloc after start-up because that can
 stall the whole device.  Its scratch is a fixed array in the library's own
 device memory instead of a caller workspace.
 
-This file is named so that pytest collects it last.  The test runs the new
-entry point twice in a row, on two different problems (the second smaller,
-so it runs over whatever the first left in the shared array), and requires
-every output to equal xshare_route's bit for bit, the bar the other routing
-tests use.  It must pass alone in a fresh process and after the other tests.
+This file is named so that pytest collects it last.  The first test runs
+the entry point on several problems in a row (each runs over whatever the
+one before left in the shared array), among them problems at the size limit
+(B = 1024 tokens, N = 1024 experts, k = 16, which reach the far ends of
+every scratch region), and requires every output to equal xshare_route's
+bit for bit, the bar the other routing tests use.  The second compares it
+with the CPU oracle directly.  They must pass alone in a fresh process and
+after the other tests.
 """
 import numpy as np
 import pytest
 import torch
 
+from oracle import xshare_oracle as O
 from paper_2602_07265_gb300 import workloads as W
 
 pytestmark = pytest.mark.gpu
@@ -50,6 +54,15 @@ def test_route_static_matches_route_twice(X):
          X.route_params(k0=1)),
         (W.random_scores(96, 128, seed=43), 8, 0, W.MODE_THRESH,
          X.route_params(k0=1, tau=0.6)),
+        # At the limit: B = 1024, N = 1024, k = 16, GROUP (Algorithms 5-6).
+        (W.random_scores(1024, 1024, seed=44), 16, 0, W.MODE_GROUP,
+         X.route_params(k0=0, n_groups=8, m_g=12)),
+        # B = 1024 with few experts (every token shares them), tie-heavy.
+        (W.random_scores(1024, 48, seed=45, ties=True), 6, 10, W.MODE_BATCH,
+         X.route_params(k0=2)),
+        # B = 1024, N = 1024, k = 16 with a warm-up set and HIER requests of 8.
+        (W.random_scores(1024, 1024, seed=46), 16, 32, W.MODE_HIER,
+         X.route_params(k0=1, m_r=2, tokens_per_request=8)),
     ]
     for p, k, budget, mode, prm in cases:
         B, N = p.shape
@@ -70,6 +83,35 @@ def test_route_static_matches_route_twice(X):
             assert np.array_equal(a.view(np.uint8), b.view(np.uint8)), key
         assert torch.equal(ref["perm"][:n_pairs].cpu(), got["perm"][:n_pairs].cpu())
         assert int(got["stats"][5].item()) == 0
+
+
+@pytest.mark.parametrize("wl", [W.DSR1, W.DSR1_GROUP.with_(B=1024)], ids=lambda w: f"{w.name}-B{w.B}")
+def test_route_static_matches_oracle(X, wl):
+    """Softmax scores the oracle computed from a seeded DeepSeek-R1-shaped
+    batch, routed by xshare_route_static and by the oracle: mask, ids,
+    weights (fp32 bits), counts, offsets, permutation and statistics equal."""
+    dev = torch.device("cuda")
+    x, W_g = W.router_inputs(wl, 3)
+    p = O.softmax_scores(O.router_logits(W.bf16_bits(x), W_g.numpy()))
+    ref = O.route(p, wl.k, wl.budget, wl.mode, **wl.params())
+    B, N, k = wl.B, wl.N, wl.k
+    got = _outputs(B, N, k, dev)
+    X.xshare_route_static(torch.from_numpy(p).to(dev), k, wl.budget, wl.mode,
+                          X.route_params(**wl.params()), got["mask"], got["ids"], got["w"],
+                          stats=got["stats"], expert_counts=got["counts"],
+                          expert_offsets=got["offsets"], perm=got["perm"])
+    torch.cuda.synchronize()
+    assert np.array_equal(got["mask"].cpu().numpy(), ref["mask"])
+    assert np.array_equal(got["ids"].cpu().numpy(), ref["ids"])
+    assert np.array_equal(got["w"].cpu().numpy().view(np.uint32), ref["w"].view(np.uint32))
+    assert np.array_equal(got["counts"].cpu().numpy(), ref["counts"])
+    assert np.array_equal(got["offsets"].cpu().numpy(), ref["offsets"])
+    n_pairs = len(ref["perm"])
+    assert np.array_equal(got["perm"][:n_pairs].cpu().numpy(), ref["perm"])
+    st = X.stats_dict(got["stats"])
+    for key in ("n_selected", "n_used", "union_topk", "max_group_load"):
+        assert st[key] == ref[key], key
+    assert st["n_pairs"] == n_pairs and st["status"] == 0
 
 
 def test_route_static_rejects_large_batches(X):
