@@ -81,6 +81,9 @@ def parse_args(argv=None):
                     help="read the expert weights as plain [N, F, d] matrices instead of packed tiles")
     ap.add_argument("--e2e-eager", action="store_true",
                     help="end-to-end steps as eager calls instead of CUDA-graph replays")
+    ap.add_argument("--ep", action="store_true",
+                    help="expert parallelism (Sec. 5): the N experts split over the ranks, one "
+                         "layer per step on one shared batch, an all-reduce of the expert outputs")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--seed", type=int, default=0)
     return ap.parse_args(argv)
@@ -515,6 +518,119 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
     return out
 
 
+def run_gpu_ep(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
+    """Expert parallelism over the ranks (Sec. 5): every rank holds the router
+    and the packed weights of its N / world experts only; a step is one layer
+    forward on one batch shared by all ranks (routing replicated, FFN over the
+    rank's experts, NCCL all-reduce of the exchange buffer, combine)."""
+    from paper_2602_07265_gb300 import _build
+    _build.build()
+    from paper_2602_07265_gb300 import xshare as X
+
+    if w.N % world != 0:
+        raise SystemExit(f"--ep needs N % ranks == 0 (N = {w.N}, ranks = {world})")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    init_dist(world, "nccl")
+    stream = torch.cuda.current_stream()
+    xs_host = [W.router_inputs(w, args.seed + i)[0] for i in range(N_ROTATE)]
+    _, W_g = W.router_inputs(w, args.seed)
+    xs_dev = [x.to(dev) for x in xs_host]
+    W_g = W_g.to(dev)
+    lo, hi = rank * (w.N // world), (rank + 1) * (w.N // world)
+    full = X.Packed(*W.expert_weights(w, args.seed, device=str(dev)))
+    pk = full.experts(lo, hi)                      # keep this rank's experts only
+    pk.gate_up, pk.down = pk.gate_up.clone(), pk.down.clone()
+    del full
+    torch.cuda.empty_cache()
+    Ns = args.shared
+    pshared = X.Packed(*W.shared_expert_weights(w, Ns, args.seed, device=str(dev))) if Ns else None
+    prm = X.route_params(**w.params())
+    ws = torch.empty(X.xshare_workspace_size(w.B, w.N, w.k, w.d, w.F, w.mode, prm, Ns),
+                     dtype=torch.uint8, device=dev)
+    buf = X.ep_exchange_buffer(ws, w.B, w.N, w.k, w.d, w.F, w.mode, prm, Ns)
+    y = torch.empty(w.B, w.d, dtype=torch.bfloat16, device=dev)
+    K, Wm = args.steps, args.warmup
+    stats = torch.zeros(K, X.STATS_WORDS, dtype=torch.int32, device=dev)
+
+    def step(x_in, st=None):
+        X.xshare_moe_forward_ep(x_in, W_g, pk, w.k, w.budget, w.mode, prm, world, rank, ws,
+                                shared=pshared, stats=st)
+        if world > 1:
+            torch.distributed.all_reduce(buf, op=torch.distributed.ReduceOp.SUM)
+        X.xshare_ep_combine(ws, w.B, w.N, w.k, w.d, w.F, w.mode, prm, y, Ns)
+
+    for i in range(Wm):
+        step(xs_dev[i % N_ROTATE])
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize()
+    with sampler:
+        t0.record(stream)
+        for i in range(K):
+            step(xs_dev[i % N_ROTATE], stats[i])
+        t1.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    ms_total = reduce_max(t0.elapsed_time(t1), world, dev)
+    st = stats.cpu().numpy()
+    if np.any(st[:, 5] != 0):
+        raise RuntimeError(f"device status {st[:, 5].max()} (a bounded wait ran out)")
+    n_used, n_pairs = st[:, 1].astype(np.float64), st[:, 4].astype(np.float64)
+    ab = [algorithmic_bytes(w, int(n_used[i]), int(n_pairs[i]), Ns) for i in range(K)]
+    layer_bytes = float(np.mean([a["layer"] for a in ab]))
+    peaks = measured_peaks()
+    step_s = ms_total / K * 1e-3
+
+    x_pin = [x.pin_memory() for x in xs_host]
+    y_pin = torch.empty(w.B, w.d, dtype=torch.bfloat16).pin_memory()
+    x_in = torch.empty(w.B, w.d, dtype=torch.bfloat16, device=dev)
+
+    def e2e_step(i):
+        x_in.copy_(x_pin[i % N_ROTATE], non_blocking=True)
+        step(x_in)
+        y_pin.copy_(y, non_blocking=True)
+        stream.synchronize()
+
+    for i in range(Wm):
+        e2e_step(i)
+    barrier(world)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(K):
+        e2e_step(i)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    e2e_ms = reduce_max(e0.elapsed_time(e1), world, dev)
+    launches = 7 - (1 if (w.B + 31) // 32 <= 2 else 0)
+    return {
+        "metric": METRIC, "value": w.B * K / (ms_total * 1e-3), "unit": "tokens/s",
+        "n_gpus": world, "steps": K, "warmup": Wm, "ms_per_step": ms_total / K,
+        "higher_is_better": True, "scaling": "strong", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic",
+        "config": dict(workload_config(w, Ns, 1),
+                       parallelism=f"expert parallel x{world} (N / {world} experts per GPU)"),
+        "experts": {"selected_mean": float(st[:, 0].mean()), "used_mean": float(n_used.mean()),
+                    "union_topk_mean": float(st[:, 2].mean()),
+                    "max_group_load_mean": float(st[:, 3].mean())},
+        "layer": {"roofline_frac": layer_bytes / world / (peaks["hbm_gbs"] * 1e9) / step_s,
+                  "note": "per-GPU share of the layer's bytes (balanced groups assumed)",
+                  "peak_source": peaks["source"]},
+        "roofline": {"kernel": "layer (expert-parallel step)", "bound": "hbm",
+                     "achieved": layer_bytes / world / step_s / 1e9, "peak": peaks["hbm_gbs"],
+                     "unit": "GB/s", "frac": layer_bytes / world / step_s / 1e9 / peaks["hbm_gbs"],
+                     "traffic": None},
+        "clocks": sampler.summary(),
+        "e2e": {"value": w.B * K / (e2e_ms * 1e-3), "unit": "tokens/s",
+                "h2d_bytes_per_step": w.B * w.d * 2, "d2h_bytes_per_step": w.B * w.d * 2},
+        "gpu_launches": launches * K,
+    }
+
+
 def run_gpu_stack(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
     """L residual layers (xshare_stack_graph_*): one step = one graph replay."""
     from paper_2602_07265_gb300 import _build
@@ -751,6 +867,13 @@ def main(argv=None):
         if rank != 0:
             return 0
         print(json.dumps(run_reference(args, w, rank, world)))
+        return 0
+    if args.ep:
+        out = run_gpu_ep(args, w, rank, world, local)
+        if rank == 0:
+            print(json.dumps(out))
+        if world > 1:
+            torch.distributed.destroy_process_group()
         return 0
     if args.layers > 1:
         out = run_gpu_stack(args, w, rank, world, local)

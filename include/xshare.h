@@ -38,8 +38,10 @@
  * Entry points: xshare_route (selection and refinement on given scores) and
  * its workspace-free variant; xshare_moe_forward (the whole layer), on plain
  * or packed expert weights (xshare_pack_experts), with optional per-kernel
- * events; xshare_stack_forward and its CUDA-graph form (L layers under one
- * global budget); a bounded-wait self-test; strings.
+ * events; its expert-parallel form over several GPUs (xshare_moe_forward_ep,
+ * xshare_ep_exchange_buffer, xshare_ep_combine); xshare_stack_forward and its
+ * CUDA-graph form (L layers under one global budget); a bounded-wait
+ * self-test; strings.
  */
 #ifndef XSHARE_H
 #define XSHARE_H
@@ -285,6 +287,54 @@ int xshare_moe_forward_packed(const uint16_t *x, const float *W_g, const xs_pack
                               uint16_t *y, float *scores_out, uint8_t *sel_mask, int32_t *topk_ids,
                               float *topk_w, xs_stats *stats, void *workspace, size_t ws_bytes,
                               xs_stream_t stream, void *const *stage_events);
+
+/* Expert parallelism (Sec. 5, Eq. 5; Algorithms 5-6 choose S so that each
+ * group's load is bounded): the N routed experts are split into n_ranks
+ * contiguous groups E_g of N / n_ranks experts, one per GPU, and rank g holds
+ * only the weights of E_g.  One layer forward over the ranks is, on every
+ * rank (one process per GPU, each with its own workspace):
+ *
+ *   1. xshare_moe_forward_ep: router, selection, refinement and permutation
+ *      over the whole batch (identical on every rank: every rank has all of x
+ *      and W_g, and the kernels are deterministic), then the SwiGLU FFN of the
+ *      (token, slot) pairs routed to E_g (and of the shared experts on rank
+ *      0) into the rank's exchange buffer, whose other rows it sets to zero;
+ *   2. the caller sums the exchange buffers of all ranks in place (an
+ *      all-reduce, e.g. ncclAllReduce with ncclSum on `stream`): every row is
+ *      non-zero on exactly one rank, so the sum is exact in any order;
+ *   3. xshare_ep_combine: the weighted combine into y, as in
+ *      xshare_moe_forward.
+ *
+ * xshare_moe_forward_ep
+ *   local_experts  the packed weights (xshare_pack_experts) of the
+ *                  local_experts->n == N / n_ranks experts of group `rank`:
+ *                  experts rank * N / n_ranks ... (rank + 1) * N / n_ranks - 1.
+ *   shared         nullable: the packed shared experts; the same count on every
+ *                  rank, their weights read on rank 0 only (other ranks may pass
+ *                  NULL pointers).
+ *   n_ranks, rank  1 <= n_ranks, N % n_ranks == 0, 0 <= rank < n_ranks.
+ *   sel_mask, topk_ids, topk_w, stats: as in xshare_moe_forward (nullable).
+ *   Other arguments and the workspace as in xshare_moe_forward_packed.
+ * xshare_ep_exchange_buffer: *buf = the exchange buffer inside `workspace`
+ *   (device, fp32, *count = (B k + n_shared B) d floats: the expert output of
+ *   every routed pair and shared row); the arguments are those of the forward.
+ *   No GPU work.
+ * xshare_ep_combine: y [B, d] bf16, device, out: the layer output from the
+ *   summed exchange buffer and the routing the forward left in `workspace`;
+ *   asynchronous on `stream`.
+ * A rank's buffer holds its own rows as fp32 values of the rank's own FFN
+ * schedule (a unit's K range may be split differently than on one GPU), so y
+ * agrees with xshare_moe_forward_packed within the forward's tolerance rather
+ * than bit for bit; with n_ranks == 1 it is identical. */
+int xshare_moe_forward_ep(const uint16_t *x, const float *W_g, const xs_packed_experts *local_experts,
+                          int B, int d, int F, int N, int k, int budget, int mode,
+                          const xs_route_params *prm, const xs_packed_experts *shared, int n_ranks,
+                          int rank, uint8_t *sel_mask, int32_t *topk_ids, float *topk_w,
+                          xs_stats *stats, void *workspace, size_t ws_bytes, xs_stream_t stream);
+int xshare_ep_exchange_buffer(void *workspace, int B, int N, int k, int d, int F, int mode,
+                              const xs_route_params *prm, int n_shared, float **buf, size_t *count);
+int xshare_ep_combine(void *workspace, int B, int N, int k, int d, int F, int mode,
+                      const xs_route_params *prm, int n_shared, uint16_t *y, xs_stream_t stream);
 
 /* Name of stage i of xshare_moe_forward (e.g. "router"), or "" if out of range. */
 const char *xshare_stage_name(int i);

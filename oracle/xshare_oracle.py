@@ -26,6 +26,8 @@ What it computes, in the paper's order and notation:
   weighted combine y = sum_i g_i(x) E_i(x) + sum_j E^s_j(x)   (Sec. 2.1)
 * A stack of L residual MoE layers with the global budget split m_l = K / L
                                                             (Eq. 1, Sec. 3.2)
+* Expert parallelism: the experts partitioned into G contiguous groups, one
+  per device, each device computing its group's pairs    (Sec. 5)
 
 Precision.  Selection is decided on fp32 scores (the precision the kernels
 decide in): softmax is evaluated in fp64 and rounded to fp32 once, column sums
@@ -608,6 +610,81 @@ def moe_forward(x_bits: np.ndarray, W_g: np.ndarray, get_expert, k: int, budget:
         y = y + shared_experts_out(x_bits, get_shared, n_shared, toks)
     r["y"] = y
     return r
+
+
+# --------------------------------------------------------------------------
+# Sec. 5: expert parallelism (experts partitioned over G devices)
+# --------------------------------------------------------------------------
+
+def expert_group_range(N: int, G: int, g: int) -> Tuple[int, int]:
+    """E_g = experts [g N/G, (g+1) N/G): G contiguous groups of N/G (N % G == 0),
+    the same partition as the groups of Algorithm 5."""
+    if N % G != 0 or not 0 <= g < G:
+        raise ValueError("need N % G == 0 and 0 <= g < G")
+    return g * (N // G), (g + 1) * (N // G)
+
+
+def moe_forward_ep_rank(x_bits: np.ndarray, W_g: np.ndarray, get_local_expert, k: int,
+                        budget: int, mode: int, G: int, g: int, get_shared=None,
+                        n_shared: int = 0, **params) -> Dict[str, object]:
+    """Device g's part of an expert-parallel layer forward (Sec. 5).
+
+    Every device holds the whole batch and the router, so the routing (router,
+    softmax, selection, refinement, permutation) is the one of `route`, the
+    same on every device.  Device g holds only the experts of E_g
+    (get_local_expert(e) for e in E_g) and computes the expert outputs of the
+    (token, slot) pairs routed to them; device 0 also computes the shared
+    experts.  They are returned as rows of an exchange matrix in the
+    permutation's order: row offsets[e] + i is the i-th pair of expert e
+    (perm), row n_pairs + j B + t is token t through shared expert j; rows of
+    other devices' experts are zero.  Summing the devices' matrices gives every
+    row from exactly one device.  Returns the routing dictionary plus "h", "p"
+    and "out" [n_pairs + n_shared B, d] float64.
+    """
+    h = router_logits(x_bits, W_g)
+    p = softmax_scores(h)
+    r = route(p, k, budget, mode, **params)
+    r["h"] = h
+    r["p"] = p
+    B, d = x_bits.shape
+    N = np.asarray(W_g).shape[0]
+    lo, hi = expert_group_range(N, G, g)
+    n_pairs = len(r["perm"])
+    out = np.zeros((n_pairs + n_shared * B, d), dtype=np.float64)
+    x = bf16_bits_to_f64(x_bits)
+    for e in range(lo, hi):
+        a, b = int(r["offsets"][e]), int(r["offsets"][e + 1])
+        if b > a:
+            tokens = [int(q) // k for q in r["perm"][a:b]]
+            Wg, Wu, Wd = get_local_expert(e)
+            out[a:b] = expert_ffn(x[tokens], Wg, Wu, Wd)
+    if g == 0:
+        for j in range(n_shared):
+            Sg, Su, Sd = get_shared(j)
+            out[n_pairs + j * B:n_pairs + (j + 1) * B] = expert_ffn(x, Sg, Su, Sd)
+    r["out"] = out
+    return r
+
+
+def ep_combine(r: Dict[str, object], out: np.ndarray, n_shared: int = 0) -> np.ndarray:
+    """The layer output from the summed exchange rows (Sec. 2.1): y_t = sum over
+    slots, in slot order, of w_ts times the row of pair (t, s), plus the sum
+    over shared experts j, in order, of row n_pairs + j B + t.  fp64."""
+    ids, w, perm = r["ids"], r["w"], r["perm"]
+    B, k = ids.shape
+    n_pairs = len(perm)
+    row_of = {int(q): i for i, q in enumerate(perm)}
+    y = np.zeros((B, out.shape[1]), dtype=np.float64)
+    for t in range(B):
+        for s in range(k):
+            if ids[t, s] >= 0:
+                y[t] += float(w[t, s]) * out[row_of[t * k + s]]
+    if n_shared:
+        sh = np.zeros_like(y)
+        for j in range(n_shared):
+            sh += out[n_pairs + j * B:n_pairs + (j + 1) * B]
+        y = y + sh
+    return y
 
 
 # --------------------------------------------------------------------------

@@ -202,9 +202,10 @@ int xs::forward_impl(const FwdCall &c, FwdStep step) {
   rc = check_ffn_shape(d, F);
   if (rc != XS_OK) return rc;
   const bool packed = c.P_gate_up != nullptr || c.P_down != nullptr;
-  if (!c.x || !c.W_g || !c.y) return XS_ERR_NULL;
+  const bool ep = c.ep_ranks >= 1;  // expert parallelism: this rank's FFN, no combine
+  if (!c.x || !c.W_g || (!ep && !c.y)) return XS_ERR_NULL;
   if (packed ? (!c.P_gate_up || !c.P_down) : (!c.W_gate || !c.W_up || !c.W_down)) return XS_ERR_NULL;
-  if (!aligned16(c.x) || !aligned16(c.W_g) || !aligned16(c.y) ||
+  if (!aligned16(c.x) || !aligned16(c.W_g) || (c.y && !aligned16(c.y)) ||
       (c.scores_out && !aligned16(c.scores_out)) || (c.resid && !aligned16(c.resid)))
     return XS_ERR_ALIGN;
   if (packed ? (!aligned16(c.P_gate_up) || !aligned16(c.P_down))
@@ -220,7 +221,8 @@ int xs::forward_impl(const FwdCall &c, FwdStep step) {
     if (!aligned16(shared->W_gate) || !aligned16(shared->W_up) || !aligned16(shared->W_down))
       return XS_ERR_ALIGN;
   }
-  if (n_shared > 0 && packed) {
+  // Under expert parallelism only rank 0 computes (and reads) the shared experts.
+  if (n_shared > 0 && packed && (!ep || c.ep_rank == 0)) {
     if (!pshared->gate_up || !pshared->down) return XS_ERR_NULL;
     if (!aligned16(pshared->gate_up) || !aligned16(pshared->down)) return XS_ERR_ALIGN;
   }
@@ -241,7 +243,14 @@ int xs::forward_impl(const FwdCall &c, FwdStep step) {
   if (c.scores_out) a.p = c.scores_out;
   if (c.sel_mask) a.mask = c.sel_mask;
   if (c.topk_ids) a.ids = c.topk_ids;
-  if (c.topk_w) a.w = c.topk_w;
+  // Under expert parallelism the weights stay in the workspace for the
+  // combine that follows the exchange (xshare_ep_combine); they are copied
+  // out afterwards if asked for.
+  if (c.topk_w && !ep) a.w = c.topk_w;
+  if (ep) {
+    a.ep_ranks = c.ep_ranks;
+    a.ep_rank = c.ep_rank;
+  }
   a.stats = c.stats;
   a.zero_words = at<int32_t>(workspace, pl.ffn_cnt);
   a.zero_count = (int)ffn_cnt_words(pl.max_tiles, B, d, F);
@@ -277,6 +286,7 @@ int xs::forward_impl(const FwdCall &c, FwdStep step) {
   f.max_rows = pl.max_rows;
   f.max_tiles = pl.max_tiles;
   f.n_sms = sms;
+  f.expert_base = ep ? c.ep_rank * (N / c.ep_ranks) : 0;
 
   auto mark = [&](int i) {
     return events == nullptr ||
@@ -296,12 +306,19 @@ int xs::forward_impl(const FwdCall &c, FwdStep step) {
   if (re != cudaSuccess || !mark(1)) return XS_ERR_CUDA;
   a.events = events ? events + 2 : nullptr;  // between the selection and refinement kernels
   if (launch_route(a, s) != cudaSuccess || !mark(3)) return XS_ERR_CUDA;
-  if (launch_gather(c.x, a.perm, a.meta, const_cast<uint16_t *>(f.xp), pl.max_rows, B, d, k,
-                    s) != cudaSuccess ||
+  if (launch_gather(c.x, a.perm, a.meta, const_cast<uint16_t *>(f.xp), ep ? f.out : nullptr,
+                    pl.max_rows, B, d, k, s) != cudaSuccess ||
       !mark(4))
     return XS_ERR_CUDA;
   if (launch_ffn_gate_up(f, s) != cudaSuccess || !mark(5)) return XS_ERR_CUDA;
   if (launch_ffn_down(f, s) != cudaSuccess || !mark(6)) return XS_ERR_CUDA;
+  if (ep) {
+    if (c.topk_w != nullptr &&
+        cudaMemcpyAsync(c.topk_w, a.w, static_cast<size_t>(B) * k * sizeof(float),
+                        cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+      return XS_ERR_CUDA;
+    return XS_OK;
+  }
   if (launch_combine(f.out, a.pos, a.w, a.meta, c.resid, c.y, B, d, k, n_shared, s) !=
           cudaSuccess ||
       !mark(7))
@@ -419,6 +436,76 @@ extern "C" int xshare_pack_experts(const uint16_t *W_gate, const uint16_t *W_up,
       launch_pack(W_down, nullptr, down, n, d, F, sms, s) != cudaSuccess)
     return XS_ERR_CUDA;
   return XS_OK;
+}
+
+extern "C" int xshare_moe_forward_ep(const uint16_t *x, const float *W_g,
+                                     const xs_packed_experts *local_experts, int B, int d, int F,
+                                     int N, int k, int budget, int mode,
+                                     const xs_route_params *prm, const xs_packed_experts *shared,
+                                     int n_ranks, int rank, uint8_t *sel_mask, int32_t *topk_ids,
+                                     float *topk_w, xs_stats *stats, void *workspace,
+                                     size_t ws_bytes, xs_stream_t stream) {
+  if (n_ranks < 1 || n_ranks > kMaxN || rank < 0 || rank >= n_ranks) return XS_ERR_PARAM;
+  if (N < 1 || N % n_ranks != 0) return XS_ERR_PARAM;
+  if (local_experts == nullptr || local_experts->gate_up == nullptr || local_experts->down == nullptr)
+    return XS_ERR_NULL;
+  if (local_experts->n != N / n_ranks) return XS_ERR_SHAPE;
+  FwdCall c = make_call(x, W_g, nullptr, nullptr, nullptr, B, d, F, N, k, budget, mode, prm, nullptr,
+                        nullptr, nullptr, sel_mask, topk_ids, topk_w, stats, workspace, ws_bytes,
+                        stream, nullptr);
+  c.P_gate_up = local_experts->gate_up;
+  c.P_down = local_experts->down;
+  c.packed_shared = shared;
+  c.ep_ranks = n_ranks;
+  c.ep_rank = rank;
+  return forward_impl(c, FwdStep::kLaunch);
+}
+
+namespace {
+
+// The plan of a forward call's workspace, after the checks xshare_ep_* share.
+int ep_plan(void *workspace, int B, int N, int k, int d, int F, int mode, const xs_route_params *prm,
+            int n_shared, Plan *pl) {
+  int rc = check_route_args(B, N, k, 0, mode, prm);
+  if (rc != XS_OK) return rc;
+  rc = check_ffn_shape(d, F);
+  if (rc != XS_OK) return rc;
+  if (n_shared < 0 || n_shared > kMaxShared) return XS_ERR_PARAM;
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return XS_ERR_WORKSPACE;
+  const int sms = current_device_sms();
+  if (sms < 0) return sms;
+  *pl = make_plan(B, N, k, d, F, true, sms, n_shared);
+  return XS_OK;
+}
+
+}  // namespace
+
+extern "C" int xshare_ep_exchange_buffer(void *workspace, int B, int N, int k, int d, int F,
+                                         int mode, const xs_route_params *prm, int n_shared,
+                                         float **buf, size_t *count) {
+  if (buf == nullptr || count == nullptr) return XS_ERR_NULL;
+  Plan pl;
+  const int rc = ep_plan(workspace, B, N, k, d, F, mode, prm, n_shared, &pl);
+  if (rc != XS_OK) return rc;
+  *buf = at<float>(workspace, pl.out);
+  *count = static_cast<size_t>(pl.max_rows) * d;
+  return XS_OK;
+}
+
+extern "C" int xshare_ep_combine(void *workspace, int B, int N, int k, int d, int F, int mode,
+                                 const xs_route_params *prm, int n_shared, uint16_t *y,
+                                 xs_stream_t stream) {
+  if (y == nullptr) return XS_ERR_NULL;
+  if (!aligned16(y)) return XS_ERR_ALIGN;
+  Plan pl;
+  const int rc = ep_plan(workspace, B, N, k, d, F, mode, prm, n_shared, &pl);
+  if (rc != XS_OK) return rc;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return launch_combine(at<float>(workspace, pl.out), at<int32_t>(workspace, pl.pos),
+                        at<float>(workspace, pl.w), at<Meta>(workspace, pl.meta), nullptr, y, B, d,
+                        k, n_shared, s) == cudaSuccess
+             ? XS_OK
+             : XS_ERR_CUDA;
 }
 
 extern "C" const char *xshare_stage_name(int i) {

@@ -84,7 +84,24 @@ struct TcParams {
   int grid;
   int n_routed;         // N: tiles of experts >= N use tmS0 / tmS1
   int has_shared;
+  int expert_base;      // routed expert e uses weights e - expert_base (expert parallelism)
 };
+
+// The FFN work of the call (Meta): routed tiles [t0, t1) then shared tiles
+// [s0, s1); work tile i is tile tile(i).
+struct WorkTiles {
+  int t0, n_routed, s0, n;
+  __device__ int tile(int i) const { return i < n_routed ? t0 + i : s0 + (i - n_routed); }
+};
+
+__device__ __forceinline__ WorkTiles work_tiles(const Meta *m) {
+  WorkTiles w;
+  w.t0 = __ldcg(&m->ffn_t0);
+  w.n_routed = __ldcg(&m->ffn_t1) - w.t0;
+  w.s0 = __ldcg(&m->ffn_s0);
+  w.n = w.n_routed + (__ldcg(&m->ffn_s1) - w.s0);
+  return w;
+}
 
 struct Range {
   long long I;      // total K steps
@@ -131,7 +148,8 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
   // own pdl_wait()), so they may be read here through L2 before pdl_wait();
   // only the token operand and the outputs depend on the kernel just before.
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n_tiles = __ldcg(&p.meta->n_tiles);
+  const WorkTiles wt = work_tiles(p.meta);
+  const int n_tiles = wt.n;
   const int MT = p.M / kBM, KI = p.K / kBK;
   Range rg;
   rg.KI = KI;
@@ -187,7 +205,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
   // Before pdl_wait() the tile is read through L2 only; after it, with a
   // plain load that also leaves it in L1 for the MMA and epilogue warps.
   auto src_of = [&](long long u, bool early) {
-    const int4 *tp = reinterpret_cast<const int4 *>(p.tiles) + u / MT;
+    const int4 *tp = reinterpret_cast<const int4 *>(p.tiles) + wt.tile(static_cast<int>(u / MT));
     const int4 t4 = early ? __ldcg(tp) : *tp;
     Src r;
     r.ntok = t4.z;
@@ -199,7 +217,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
     const bool routed = t4.x < p.n_routed;
     r.mA0 = routed ? &p.tmA0 : &p.tmS0;
     r.mA1 = routed ? &p.tmA1 : &p.tmS1;
-    const int e_local = routed ? t4.x : t4.x - p.n_routed;
+    const int e_local = routed ? t4.x - p.expert_base : t4.x - p.n_routed;
     r.arow = e_local * p.M + mt * kBM;
     r.pblk = p.pk ? (routed ? p.pk : p.pk_shared) +
                         ((static_cast<size_t>(e_local) * MT + mt) * KI) * (C::kNumA * kTileBytes)
@@ -317,7 +335,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
         const long long u = it / KI;
         const int k0 = static_cast<int>(it - u * KI);
         const int k1 = static_cast<int>(k0 + (it_end - it) < KI ? k0 + (it_end - it) : KI);
-        const Tile tl = p.tiles[u / MT];
+        const Tile tl = p.tiles[wt.tile(static_cast<int>(u / MT))];
         const int n_mma = ((tl.ntok + 15) / 16) * 16;
         const uint32_t idesc = idesc_bf16(kBM, n_mma);
         const int buf = segi & 1;
@@ -374,7 +392,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
       const long long u = it / KI;
       const int k0 = static_cast<int>(it - u * KI);
       const int k1 = static_cast<int>(k0 + (it_end - it) < KI ? k0 + (it_end - it) : KI);
-      const Tile tl = p.tiles[u / MT];
+      const Tile tl = p.tiles[wt.tile(static_cast<int>(u / MT))];
       const int mt = static_cast<int>(u % MT);
       const int n_mma = ((tl.ntok + 15) / 16) * 16;
       const int buf = segi & 1;
@@ -532,6 +550,7 @@ cudaError_t launch_ffn_gate_up(const FfnArgs &a, cudaStream_t s) {
   }
   p.n_routed = a.N;
   p.has_shared = a.n_shared > 0;
+  p.expert_base = a.expert_base;
   p.tiles = a.tiles;
   p.meta = a.meta;
   p.stats = a.stats;
@@ -565,6 +584,7 @@ cudaError_t launch_ffn_down(const FfnArgs &a, cudaStream_t s) {
   p.tmS1 = p.tmS0;
   p.n_routed = a.N;
   p.has_shared = a.n_shared > 0;
+  p.expert_base = a.expert_base;
   p.tiles = a.tiles;
   p.meta = a.meta;
   p.stats = a.stats;

@@ -292,6 +292,11 @@ __device__ __forceinline__ void selection_stats(const RouteArgs &a, const uint8_
                                                 int &nsel, int &maxload) {
   const int tid = threadIdx.x, N = a.N;
   const int G = a.G >= 1 ? a.G : 1, size = N / G;
+  if (G == 1) {  // one group: its load is |S|
+    nsel = __syncthreads_count(tid < N && s_mask[tid]);
+    maxload = nsel;
+    return;
+  }
   for (int g = tid; g < G; g += blockDim.x) s_gl[g] = 0;
   __syncthreads();
   for (int j = tid; j < N; j += blockDim.x)
@@ -466,6 +471,32 @@ __device__ void build_permutation(const RouteArgs &a, PermSmem sm) {
       sm.scal[1] = tot[0];  // pairs
       sm.scal[2] = tot[1];  // tiles
       sm.scal[3] = tot[2];  // used experts
+    }
+    // This call's FFN work (Sec. 5): the tiles and rows of the experts of
+    // group ep_rank, a contiguous index range, hence contiguous tiles and
+    // rows; shared experts go to rank 0.  Without expert parallelism: all.
+    {
+      const int G = a.ep_ranks > 1 ? a.ep_ranks : 1, g = G > 1 ? a.ep_rank : 0;
+      const int e_lo = g * (N / G), e_hi = (g + 1) * (N / G);
+      Meta *m = a.meta;
+      if (tid == e_lo) {
+        m->ffn_t0 = v[1];
+        m->row0 = v[0];
+      }
+      if (e_hi < N && tid == e_hi) {
+        m->ffn_t1 = v[1];
+        m->row1 = v[0];
+      }
+      if (tid == 0) {
+        if (e_hi >= N) {
+          m->ffn_t1 = tot[1];
+          m->row1 = tot[0];
+        }
+        const int own_shared = g == 0 ? 1 : 0;
+        m->ffn_s0 = tot[1];
+        m->ffn_s1 = tot[1] + own_shared * a.n_shared * ((B + kTileTok - 1) / kTileTok);
+        m->srows = own_shared;
+      }
     }
     // Shared experts: every token, in token order, after the routed pairs.
     const int tpt = (B + kTileTok - 1) / kTileTok;
@@ -1104,17 +1135,28 @@ __global__ void __launch_bounds__(kRtWarps * 32) router_logits_kernel(
   }
 }
 
-// Xp[row] = x[token of pair perm[row]], 16-byte vectors.
+// Xp[row] = x[token of pair perm[row]], 16-byte vectors, for the rows this
+// call's FFN computes; with expert parallelism the other rows of zero_out
+// (computed by other ranks) are set to zero instead.
 __global__ void __launch_bounds__(256) gather_kernel(const uint16_t *__restrict__ x,
                                                      const int32_t *__restrict__ perm,
                                                      const Meta *__restrict__ meta,
-                                                     uint16_t *__restrict__ xp, int B, int d,
+                                                     uint16_t *__restrict__ xp,
+                                                     float *__restrict__ zero_out, int B, int d,
                                                      int k) {
   pdl_wait();
   pdl_trigger();
   const int row = blockIdx.x;
   const int P = meta->n_pairs;
   if (row >= meta->n_rows) return;
+  const bool mine = row < P ? (row >= meta->row0 && row < meta->row1) : meta->srows != 0;
+  if (!mine) {
+    if (zero_out != nullptr) {
+      float4 *dst = reinterpret_cast<float4 *>(zero_out + static_cast<size_t>(row) * d);
+      for (int i = threadIdx.x; i < d / 4; i += blockDim.x) dst[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    return;
+  }
   const int t = row < P ? perm[row] / k : (row - P) % B;  // routed pair, else shared row
   const uint4 *src = reinterpret_cast<const uint4 *>(x + (size_t)t * d);
   uint4 *dst = reinterpret_cast<uint4 *>(xp + (size_t)row * d);
@@ -1230,8 +1272,10 @@ cudaError_t launch_router_logits(const uint16_t *x, const float *Wg, float *h, i
 }
 
 cudaError_t launch_gather(const uint16_t *x, const int32_t *perm, const Meta *meta,
-                          uint16_t *xp, int max_rows, int B, int d, int k, cudaStream_t s) {
-  return launch_pdl(gather_kernel, dim3(max_rows), dim3(256), 0, s, x, perm, meta, xp, B, d, k);
+                          uint16_t *xp, float *zero_out, int max_rows, int B, int d, int k,
+                          cudaStream_t s) {
+  return launch_pdl(gather_kernel, dim3(max_rows), dim3(256), 0, s, x, perm, meta, xp, zero_out, B,
+                    d, k);
 }
 
 cudaError_t launch_combine(const float *out, const int32_t *pos, const float *w,

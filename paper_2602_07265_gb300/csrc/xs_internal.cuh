@@ -76,7 +76,12 @@ struct Meta {
   int32_t max_group_load;
   int32_t status;       // XS_DEV_*
   int32_t n_rows;       // FFN rows: n_pairs + n_shared * B
-  int32_t pad[7];
+  // The FFN work of this call: routed tiles [ffn_t0, ffn_t1) and shared-expert
+  // tiles [ffn_s0, ffn_s1), in that order; the rows they write: routed rows
+  // [row0, row1) and, if srows, the shared rows.  Without expert parallelism
+  // that is every tile and row; with it, those of the rank's expert group.
+  int32_t ffn_t0, ffn_t1, ffn_s0, ffn_s1;
+  int32_t row0, row1, srows;
 };
 
 // Byte offsets of every workspace region (256-byte aligned).
@@ -123,6 +128,7 @@ struct RouteArgs {
   int n_shared;          // shared-expert tiles appended after the routed ones
   const int32_t *router_status;  // nullable: per-CTA status of the tensor-core router
   int router_ctas;
+  int ep_ranks, ep_rank;  // expert parallelism: the FFN work of group ep_rank of ep_ranks (0: all)
 };
 
 cudaError_t launch_route(const RouteArgs &a, cudaStream_t s);
@@ -138,8 +144,12 @@ cudaError_t launch_router_tc(const uint16_t *x, const float *Wg, float *h, int B
 cudaError_t launch_combine(const float *out, const int32_t *pos, const float *w,
                            const Meta *meta, const uint16_t *resid, uint16_t *y, int B, int d,
                            int k, int n_shared, cudaStream_t s);
+// Gathers the token rows of this call's FFN rows into xp; with expert
+// parallelism (zero_out != nullptr) it zeroes the rows of zero_out that
+// another rank computes.
 cudaError_t launch_gather(const uint16_t *x, const int32_t *perm, const Meta *meta,
-                          uint16_t *xp, int max_rows, int B, int d, int k, cudaStream_t s);
+                          uint16_t *xp, float *zero_out, int max_rows, int B, int d, int k,
+                          cudaStream_t s);
 
 struct FfnArgs {
   const uint16_t *W_gate, *W_up, *W_down;
@@ -156,6 +166,7 @@ struct FfnArgs {
   void *part;            // partial-sum scratch
   int32_t *cnt;          // arrival counters (cleared by the routing kernel)
   int N, d, F, max_rows, max_tiles, n_sms;
+  int expert_base;       // routed expert e uses weights e - expert_base (expert parallelism)
 };
 
 cudaError_t launch_ffn_gate_up(const FfnArgs &a, cudaStream_t s);
@@ -188,6 +199,7 @@ struct FwdCall {
   size_t ws_bytes;
   xs_stream_t stream;
   void *const *events;
+  int ep_ranks, ep_rank;  // > 1: expert parallelism; the call ends after the FFN (no combine)
 };
 
 enum class FwdStep {

@@ -93,6 +93,14 @@ def _load() -> ctypes.CDLL:
     lib.xshare_moe_forward_packed.argtypes = [P, P, PP, I, I, I, I, I, I, I, PR, PP,
                                               P, P, P, P, P, P, P, Z, P, P]
     lib.xshare_moe_forward_packed.restype = I
+    lib.xshare_moe_forward_ep.argtypes = [P, P, PP, I, I, I, I, I, I, I, PR, PP, I, I,
+                                          P, P, P, P, P, Z, P]
+    lib.xshare_moe_forward_ep.restype = I
+    lib.xshare_ep_exchange_buffer.argtypes = [P, I, I, I, I, I, I, PR, I, ctypes.POINTER(P),
+                                              ctypes.POINTER(Z)]
+    lib.xshare_ep_exchange_buffer.restype = I
+    lib.xshare_ep_combine.argtypes = [P, I, I, I, I, I, I, PR, I, P, P]
+    lib.xshare_ep_combine.restype = I
     PL = ctypes.POINTER(Layer)
     lib.xshare_stack_forward.argtypes = [P, PL, I, I, I, I, I, I, I, I, PR, P, P, P, Z, P]
     lib.xshare_stack_forward.restype = I
@@ -274,6 +282,18 @@ class Packed:
     def struct(self) -> PackedExperts:
         return PackedExperts(self.gate_up.data_ptr(), self.down.data_ptr(), self.n)
 
+    def experts(self, lo: int, hi: int) -> "Packed":
+        """Experts lo .. hi-1 as packed weights of their own (views of these
+        buffers: the packed layout keeps each expert's tiles contiguous)."""
+        if not 0 <= lo < hi <= self.n:
+            raise ValueError(f"expert range [{lo}, {hi}) outside [0, {self.n})")
+        v = Packed.__new__(Packed)
+        v.n, v.d, v.F = hi - lo, self.d, self.F
+        gu, dn = self.F * self.d * 2 * 2, self.d * self.F * 2
+        v.gate_up = self.gate_up[lo * gu:hi * gu]
+        v.down = self.down[lo * dn:hi * dn]
+        return v
+
 
 def xshare_moe_forward_packed(x: torch.Tensor, W_g: torch.Tensor, experts: Packed, k: int,
                               budget: int, mode: int, params: RouteParams, y: torch.Tensor,
@@ -309,6 +329,74 @@ def xshare_moe_forward_packed(x: torch.Tensor, W_g: torch.Tensor, experts: Packe
         _ptr(topk_w, torch.float32, "topk_w", B * k), _ptr(stats, torch.int32, "stats", STATS_WORDS),
         _ptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream), handles)
     _check(rc, "xshare_moe_forward_packed")
+
+
+def xshare_moe_forward_ep(x: torch.Tensor, W_g: torch.Tensor, local_experts: Packed, k: int,
+                          budget: int, mode: int, params: RouteParams, n_ranks: int, rank: int,
+                          workspace: torch.Tensor, shared: Optional[Packed] = None,
+                          sel_mask: Optional[torch.Tensor] = None,
+                          topk_ids: Optional[torch.Tensor] = None,
+                          topk_w: Optional[torch.Tensor] = None,
+                          stats: Optional[torch.Tensor] = None, stream=None) -> None:
+    """This rank's part of an expert-parallel layer forward (routing of the
+    whole batch, the FFN of expert group `rank`); see xshare.h."""
+    B, d = x.shape
+    N = W_g.shape[0]
+    if local_experts.n * n_ranks != N or local_experts.d != d or W_g.shape[1] != d:
+        raise ValueError("inconsistent shapes")
+    ex = local_experts.struct()
+    sh = shared.struct() if shared is not None else None
+    rc = LIB.xshare_moe_forward_ep(
+        _ptr(x, torch.bfloat16, "x"), _ptr(W_g, torch.float32, "W_g"), ctypes.byref(ex), B, d,
+        local_experts.F, N, k, budget, mode, ctypes.byref(params),
+        ctypes.byref(sh) if sh is not None else None, n_ranks, rank,
+        _ptr(sel_mask, torch.uint8, "sel_mask", N), _ptr(topk_ids, torch.int32, "topk_ids", B * k),
+        _ptr(topk_w, torch.float32, "topk_w", B * k), _ptr(stats, torch.int32, "stats", STATS_WORDS),
+        _ptr(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream))
+    _check(rc, "xshare_moe_forward_ep")
+
+
+def ep_exchange_buffer(workspace: torch.Tensor, B: int, N: int, k: int, d: int, F: int, mode: int,
+                       params: RouteParams, n_shared: int = 0) -> torch.Tensor:
+    """The exchange buffer of an expert-parallel forward: an fp32 view of the
+    workspace (xshare_ep_exchange_buffer)."""
+    buf, count = ctypes.c_void_p(), ctypes.c_size_t()
+    _check(LIB.xshare_ep_exchange_buffer(_ptr(workspace, torch.uint8, "workspace"), B, N, k, d, F,
+                                         mode, ctypes.byref(params), n_shared, ctypes.byref(buf),
+                                         ctypes.byref(count)), "xshare_ep_exchange_buffer")
+    off = buf.value - workspace.data_ptr()
+    if off < 0 or off + 4 * count.value > workspace.numel():
+        raise XShareError(-4, "ep_exchange_buffer")
+    return workspace[off:off + 4 * count.value].view(torch.float32)
+
+
+def xshare_ep_combine(workspace: torch.Tensor, B: int, N: int, k: int, d: int, F: int, mode: int,
+                      params: RouteParams, y: torch.Tensor, n_shared: int = 0, stream=None) -> None:
+    """The weighted combine after the exchange; see xshare.h."""
+    if tuple(y.shape) != (B, d):
+        raise ValueError("y must be [B, d]")
+    _check(LIB.xshare_ep_combine(_ptr(workspace, torch.uint8, "workspace"), B, N, k, d, F, mode,
+                                 ctypes.byref(params), n_shared, _ptr(y, torch.bfloat16, "y"),
+                                 _stream(stream)), "xshare_ep_combine")
+
+
+def ep_layer_forward(x: torch.Tensor, W_g: torch.Tensor, local_experts: Packed, k: int,
+                     budget: int, mode: int, params: RouteParams, y: torch.Tensor,
+                     workspace: torch.Tensor, group=None, shared: Optional[Packed] = None,
+                     stats: Optional[torch.Tensor] = None, n_shared: int = 0) -> None:
+    """One expert-parallel layer forward over the ranks of a torch.distributed
+    process group (one GPU per rank): this rank's forward, an in-place sum
+    all-reduce of the exchange buffers, the combine."""
+    import torch.distributed as dist
+    n_ranks = dist.get_world_size(group)
+    rank = dist.get_rank(group)
+    B, d = x.shape
+    N = W_g.shape[0]
+    xshare_moe_forward_ep(x, W_g, local_experts, k, budget, mode, params, n_ranks, rank, workspace,
+                          shared=shared, stats=stats)
+    buf = ep_exchange_buffer(workspace, B, N, k, d, local_experts.F, mode, params, n_shared)
+    dist.all_reduce(buf, op=dist.ReduceOp.SUM, group=group)
+    xshare_ep_combine(workspace, B, N, k, d, local_experts.F, mode, params, y, n_shared)
 
 
 def _stack_args(x, layers, k, K_total, mode, params, h_out, workspace, stats):

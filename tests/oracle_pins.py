@@ -687,6 +687,51 @@ def check_sparse_selection(O, cases=30):
         assert mask_to_set(c["mask"]) <= mask_to_set(a["mask"])
 
 
+def check_expert_parallel(O):
+    """Sec. 5, experts split over G devices: device g's exchange rows hold, at
+    row offsets[e] + i, the SwiGLU output (torch float64) of the i-th pair of
+    each of its experts e, and at n_pairs + j B + t (device 0 only) token t
+    through shared expert j; all other rows are zero.  The rows of all
+    devices, summed, combine to the one-device layer output exactly."""
+    g = torch.Generator().manual_seed(21)
+    N, k, d, F, B, Ns = 8, 2, 16, 8, 5, 1
+    x = bf16_round(torch.randn(B, d, generator=g))
+    W_g = torch.randn(N, d, generator=g) / math.sqrt(d)
+    Wg = bf16_round(torch.randn(N, F, d, generator=g) * 0.2)
+    Wu = bf16_round(torch.randn(N, F, d, generator=g) * 0.2)
+    Wd = bf16_round(torch.randn(N, d, F, generator=g) * 0.2)
+    Sg = bf16_round(torch.randn(Ns, F, d, generator=g) * 0.2)
+    Su = bf16_round(torch.randn(Ns, F, d, generator=g) * 0.2)
+    Sd = bf16_round(torch.randn(Ns, d, F, generator=g) * 0.2)
+    get = lambda e: (bits(Wg[e]), bits(Wu[e]), bits(Wd[e]))
+    gets = lambda j: (bits(Sg[j]), bits(Su[j]), bits(Sd[j]))
+    X = x.to(torch.float64)
+
+    def swiglu(t, Wg_, Wu_, Wd_):
+        a = torch.nn.functional.silu(X[t] @ Wg_.to(torch.float64).T) * (X[t] @ Wu_.to(torch.float64).T)
+        return (a @ Wd_.to(torch.float64).T).numpy()
+
+    ref = O.moe_forward(bits(x), W_g.numpy(), get, k, 3, O.MODE_BATCH, get_shared=gets, n_shared=Ns)
+    for G in (2, 4):
+        total = 0
+        for dev in range(G):
+            lo, hi = (N // G) * dev, (N // G) * (dev + 1)
+            r = O.moe_forward_ep_rank(bits(x), W_g.numpy(), get, k, 3, O.MODE_BATCH, G, dev,
+                                      get_shared=gets, n_shared=Ns)
+            n_pairs = len(r["perm"])
+            for row in range(r["out"].shape[0]):
+                if row < n_pairs:
+                    q = int(r["perm"][row])
+                    e = int(r["ids"][q // k, q % k])
+                    want = swiglu(q // k, Wg[e], Wu[e], Wd[e]) if lo <= e < hi else np.zeros(d)
+                else:
+                    t = (row - n_pairs) % B
+                    want = swiglu(t, Sg[0], Su[0], Sd[0]) if dev == 0 else np.zeros(d)
+                assert np.allclose(r["out"][row], want, rtol=1e-12, atol=1e-14), (G, dev, row)
+            total = total + r["out"]
+        assert np.array_equal(O.ep_combine(ref, total, Ns), ref["y"])
+
+
 ALL_CHECKS = [
     check_closed_form_golden, check_union_statistics, check_greedy_bruteforce,
     check_hier_bruteforce, check_hier_single_request_is_batch, check_group,
@@ -695,5 +740,5 @@ ALL_CHECKS = [
     check_combine_multi_token, check_canonical_sum_golden, check_canonical_sum_bound,
     check_threshold_golden, check_threshold_bruteforce, check_threshold_consistency,
     check_bf16_rounding, check_layer_budgets, check_stack_invariants,
-    check_topk_gating, check_sparse_selection,
+    check_topk_gating, check_sparse_selection, check_expert_parallel,
 ]

@@ -27,7 +27,9 @@ def declared_functions():
 
 
 def test_header_declares_the_boundary():
-    assert declared_functions() == ["xshare_moe_forward", "xshare_moe_forward_packed",
+    assert declared_functions() == ["xshare_ep_combine", "xshare_ep_exchange_buffer",
+                                    "xshare_moe_forward", "xshare_moe_forward_ep",
+                                    "xshare_moe_forward_packed",
                                     "xshare_moe_forward_profiled", "xshare_pack_experts",
                                     "xshare_route", "xshare_route_static",
                                     "xshare_selftest_wait_timeout", "xshare_stack_forward",
@@ -170,3 +172,31 @@ def test_packed_entry_points_reject_bad_arguments(X):
     assert rc(ex=X.PackedExperts(P + 4, P, 16)) == -5
     assert rc(sh=X.PackedExperts(P, P, 9)) == -2
     assert rc(sh=X.PackedExperts(None, P, 1)) == -3
+
+
+def test_ep_entry_points_reject_bad_arguments(X):
+    """Expert-parallel calls: n_ranks and rank, N % n_ranks, the local expert
+    count, NULL outputs; all checked before anything touches a GPU."""
+    prm = X.route_params()
+    ws = ctypes.c_void_p(256)  # never dereferenced: every call below fails its checks first
+    pk = X.PackedExperts(16, 16, 32)
+
+    def fwd(n_ranks, rank, N=64, local=pk):
+        return X.LIB.xshare_moe_forward_ep(16, 16, ctypes.byref(local) if local else None, 32, 512,
+                                           256, N, 8, 24, 1, ctypes.byref(prm), None, n_ranks,
+                                           rank, None, None, None, None, ws, 1 << 30, None)
+    assert fwd(0, 0) == -2          # n_ranks < 1
+    assert fwd(2, 2) == -2          # rank >= n_ranks
+    assert fwd(2, -1) == -2         # rank < 0
+    assert fwd(3, 0) == -2          # N % n_ranks != 0
+    assert fwd(2, 0, local=None) == -3
+    assert fwd(2, 0, local=X.PackedExperts(16, 16, 16)) == -1   # N / n_ranks = 32 experts expected
+    buf, count = ctypes.c_void_p(), ctypes.c_size_t()
+    assert X.LIB.xshare_ep_exchange_buffer(ws, 32, 64, 8, 512, 256, 1, ctypes.byref(prm), 0,
+                                           None, ctypes.byref(count)) == -3
+    assert X.LIB.xshare_ep_exchange_buffer(ws, 32, 64, 8, 500, 256, 1, ctypes.byref(prm), 0,
+                                           ctypes.byref(buf), ctypes.byref(count)) == -1
+    assert X.LIB.xshare_ep_combine(ws, 32, 64, 8, 512, 256, 1, ctypes.byref(prm), 0, None,
+                                   None) == -3
+    assert X.LIB.xshare_ep_combine(ws, 32, 64, 8, 512, 256, 1, ctypes.byref(prm), 0, 18,
+                                   None) == -5

@@ -212,6 +212,26 @@ def _candidates_allow_zero(scores, S, positive_only, pool=None):
     return _orig["candidates"](scores, S, False, pool)
 
 
+def _group_range_shifted(N, G, g):
+    lo, hi = _orig["expert_group_range"](N, G, g)
+    return lo + 1, min(hi + 1, N)
+
+
+def _ep_combine_shared_first(r, out, n_shared=0):
+    ids, w, perm = r["ids"], r["w"], r["perm"]
+    B, k = ids.shape
+    n_pairs = len(perm)
+    row_of = {int(q): i for i, q in enumerate(perm)}
+    y = np.zeros((B, out.shape[1]))
+    for t in range(B):
+        for j in range(n_shared):
+            y[t] += out[n_pairs + j * B + t]
+        for s in range(k):
+            if ids[t, s] >= 0:
+                y[t] += float(w[t, s]) * out[row_of[t * k + s]]
+    return y
+
+
 def _closed_form_wrong(N, k, B):
     return N * (1.0 - (1.0 - k / N) ** (B - 1))
 
@@ -247,6 +267,8 @@ MUTATIONS = {
     "bf16 rounded through fp32": ("f64_to_bf16_bits", _bf16_via_fp32),
     "sparse gating not renormalised": ("topk_gating", _gating_unnormalised),
     "sparse selection adds zero-gain experts": ("candidates", _candidates_allow_zero),
+    "device owns the wrong expert group": ("expert_group_range", _group_range_shifted),
+    "combine adds the shared experts first": ("ep_combine", _ep_combine_shared_first),
 }
 
 _orig = {name: getattr(O, name) for name, _ in MUTATIONS.values()}
