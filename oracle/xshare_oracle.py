@@ -246,11 +246,12 @@ def expert_tree_sum(values: np.ndarray, members: Set[int]) -> np.float32:
 
 def greedy_select_threshold(scores: np.ndarray, tau: float, S0: Set[int],
                             positive_only: bool = False) -> Set[int]:
-    """Algorithm 1 as printed, with a threshold tau on the covered score mass.
+    """Algorithm 1 in its threshold form: experts are added until they cover
+    a fraction tau of the batch's score mass.
 
-    Starting from S_0, while f(S) < tau * f(E), add argmax_{e in E \\ S}
-    scores[e] (Algorithm 1's loop; its condition names P for G, read as the
-    scores G).  The loop also ends when E \\ S is empty.
+    Starting from S_0, while f(S) < tau * f(E), the expert of E \\ S with the
+    largest score is added (Algorithm 1's condition names P for G, read as the
+    scores G).  Selection also ends when E \\ S is empty.
 
     Precision.  f(E) and f(S_0) are `expert_tree_sum`s; the target is the
     fp32 product tau * f(E) rounded once.  When e is added, f(S) becomes the
@@ -330,27 +331,32 @@ def group_of(e: int, N: int, G: int) -> int:
 
 def gpu_aware_greedy(scores: np.ndarray, G: int, m_g: int, S0: Set[int],
                      positive_only: bool = False) -> Set[int]:
-    """Algorithm 5 taken literally.
+    """Algorithm 5 (Sec. 5.1): greedy selection with a per-group budget m_g
+    over the G contiguous expert groups E_g.
 
-    S = S_0; while |S| < m_g * G: for g = 1..G: add the argmax of the marginal
-    gain over E_g \\ S (the column score, by Proposition 1).
-    Readings: a round always runs over all G groups, so |S| may end above
-    m_g * G by up to G - 1; a group with nothing left is skipped; when every
-    group is exhausted the loop stops (the pseudocode would not terminate).
+    By Proposition 1 the marginal gain of adding expert e is its column score
+    scores[e], whatever has been selected, so the order in which a group
+    receives experts is known in advance: its candidates E_g \ S_0 (with a
+    positive score when positive_only) ranked by score.  Selection proceeds in
+    rounds; round r gives every group that still has an r-th candidate that
+    expert.  Rounds are whole (every group gets its turn in each), and a new
+    round starts while |S| < m_g * G and some group still has candidates.
+    Readings: |S| may therefore end above m_g * G by up to G - 1; S_0 is kept
+    even where it exceeds a group's share; selection stops when every group is
+    exhausted.
     """
     N = scores.shape[0]
     size = N // G
+    order = [ranked(scores, candidates(scores, set(S0), positive_only,
+                                       range(g * size, (g + 1) * size)))
+             for g in range(G)]
     S = set(S0)
-    while len(S) < m_g * G:
-        added = False
-        for g in range(G):
-            rest = candidates(scores, S, positive_only, range(g * size, (g + 1) * size))
-            if not rest:
-                continue
-            S.add(ranked(scores, rest)[0])
-            added = True
-        if not added:
-            break
+    r = 0
+    while len(S) < m_g * G and any(r < len(o) for o in order):
+        for o in order:
+            if r < len(o):
+                S.add(o[r])
+        r += 1
     return S
 
 

@@ -930,9 +930,9 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
         });
       }
   } else if (a.mode == XS_MODE_THRESH) {
-    // Algorithm 1 as printed: add the best remaining expert while the
-    // covered mass f(S) is below tau f(E); by Proposition 1 adding e adds
-    // scores[e] to f(S).
+    // Algorithm 1 in its threshold form: add the best remaining expert
+    // while the covered mass f(S) is below tau f(E); by Proposition 1 adding
+    // e adds scores[e] to f(S).
     if (warp == 0) {
       float vE[kQ], v0[kQ];
 #pragma unroll
