@@ -84,6 +84,11 @@ def parse_args(argv=None):
     ap.add_argument("--ep", action="store_true",
                     help="expert parallelism (Sec. 5): the N experts split over the ranks, one "
                          "layer per step on one shared batch, an all-reduce of the expert outputs")
+    ap.add_argument("--sweep", action="append", default=[], metavar="FIELD=V1,V2,...",
+                    help="sweep mode: time every combination of these workload fields (B, budget, "
+                         "k0, m_r, m_g, tau, mode, tokens_per_request, sparse_scores), one JSON line "
+                         "per combination with the median over --seeds")
+    ap.add_argument("--seeds", default="0", help="comma-separated seeds (sweep mode)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--seed", type=int, default=0)
     return ap.parse_args(argv)
@@ -631,6 +636,89 @@ def run_gpu_ep(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
     }
 
 
+def parse_sweep(specs) -> list:
+    """[(field, [values])] from FIELD=V1,V2 strings; values typed by the field."""
+    out = []
+    for spec in specs:
+        field, _, vals = spec.partition("=")
+        if field not in ("B", "budget", "k0", "m_r", "m_g", "tau", "mode", "tokens_per_request",
+                         "sparse_scores") or not vals:
+            raise SystemExit(f"bad --sweep {spec!r}")
+        conv = float if field == "tau" else (lambda v: W.MODES[v] if v in W.MODES else int(v)) \
+            if field == "mode" else int
+        out.append((field, [conv(v) for v in vals.split(",")]))
+    return out
+
+
+def run_sweep(args, w0: W.Workload) -> list:
+    """Sweep mode (one GPU): for every seed the expert weights are drawn and
+    packed once; every combination of the swept fields is timed like the
+    headline (back-to-back steps, CUDA events, rotating inputs) and reported
+    with the median over the seeds."""
+    import itertools
+    from paper_2602_07265_gb300 import _build
+    _build.build()
+    from paper_2602_07265_gb300 import xshare as X
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    fields = parse_sweep(args.sweep)
+    combos = [dict(zip([f for f, _ in fields], vals))
+              for vals in itertools.product(*[v for _, v in fields])]
+    seeds = [int(v) for v in args.seeds.split(",")]
+    peaks = measured_peaks()
+    K, Wm = args.steps, args.warmup
+    res = {i: [] for i in range(len(combos))}
+    for seed in seeds:
+        pk = X.Packed(*W.expert_weights(w0, seed, device=str(dev)))
+        torch.cuda.empty_cache()
+        for i, kw in enumerate(combos):
+            w = w0.with_(**kw)
+            # Seed 0 uses the headline's input batches (0 .. N_ROTATE - 1).
+            xs = [W.router_inputs(w, 101 * seed + j)[0].to(dev) for j in range(N_ROTATE)]
+            W_g = W.router_inputs(w, seed)[1].to(dev)
+            prm = X.route_params(**w.params())
+            ws = torch.empty(X.xshare_workspace_size(w.B, w.N, w.k, w.d, w.F, w.mode, prm, 0),
+                             dtype=torch.uint8, device=dev)
+            y = torch.empty(w.B, w.d, dtype=torch.bfloat16, device=dev)
+            st = torch.zeros(K, X.STATS_WORDS, dtype=torch.int32, device=dev)
+
+            def step(j, stats=None):
+                X.xshare_moe_forward_packed(xs[j % N_ROTATE], W_g, pk, w.k, w.budget, w.mode, prm, y,
+                                            ws, stats=stats)
+            for j in range(Wm):
+                step(j)
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for j in range(K):
+                step(j, st[j])
+            e1.record()
+            torch.cuda.synchronize()
+            s = st.cpu().numpy()
+            if np.any(s[:, 5] != 0):
+                raise RuntimeError("device status: a bounded wait ran out")
+            lb = float(np.mean([algorithmic_bytes(w, int(s[j, 1]), int(s[j, 4]))["layer"] for j in range(K)]))
+            ms = e0.elapsed_time(e1) / K
+            res[i].append({"ms": ms, "S": float(s[:, 0].mean()), "U": float(s[:, 1].mean()),
+                           "union": float(s[:, 2].mean()), "maxload": float(s[:, 3].mean()),
+                           "roofline": lb / (peaks["hbm_gbs"] * 1e9) / (ms * 1e-3)})
+        del pk
+        torch.cuda.empty_cache()
+    lines = []
+    for i, kw in enumerate(combos):
+        w = w0.with_(**kw)
+        med = {key: float(np.median([r[key] for r in res[i]])) for key in res[i][0]}
+        lines.append({"sweep": describe(w), "fields": kw, "seeds": seeds, "steps": K,
+                      "ms_per_step_median": med["ms"], "ms_per_step": [r["ms"] for r in res[i]],
+                      "tokens_per_s_median": w.B / (med["ms"] * 1e-3),
+                      "roofline_frac_median": med["roofline"],
+                      "experts_median": {"selected": med["S"], "used": med["U"],
+                                         "union_topk": med["union"], "max_group_load": med["maxload"]},
+                      "peak_source": peaks["source"]})
+    return lines
+
+
 def run_gpu_stack(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
     """L residual layers (xshare_stack_graph_*): one step = one graph replay."""
     from paper_2602_07265_gb300 import _build
@@ -867,6 +955,12 @@ def main(argv=None):
         if rank != 0:
             return 0
         print(json.dumps(run_reference(args, w, rank, world)))
+        return 0
+    if args.sweep:
+        if world > 1:
+            raise SystemExit("sweep mode runs on one GPU")
+        for line in run_sweep(args, w):
+            print(json.dumps(line), flush=True)
         return 0
     if args.ep:
         out = run_gpu_ep(args, w, rank, world, local)
