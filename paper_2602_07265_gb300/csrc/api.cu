@@ -116,7 +116,9 @@ Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms, int 
     o = align_up(o + bytes);
     return r;
   };
-  pl.h = take((size_t)B * N * 4);
+  const bool split = with_ffn && B < kRouterTcMinB && d >= kRouterSplitMinD && d <= kRouterSplitMaxD;
+  const int h_splits = split ? router_split_count(B, N, d, n_sms) : 1;
+  pl.h = take((size_t)h_splits * B * N * 4);
   pl.p = take((size_t)B * N * 4);
   pl.mask = take((size_t)N);
   pl.ids = take((size_t)B * k * 4);
@@ -134,7 +136,7 @@ Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms, int 
   pl.done = take(4 * sizeof(int32_t));
   pl.gs = take((size_t)B * N * 4);
   if (with_ffn) {
-    pl.rstat = take((size_t)router_tc_ctas(B, N, d, n_sms) * 4);
+    pl.rstat = take((size_t)(split ? router_split_ctas(B, N, d, n_sms) : router_tc_ctas(B, N, d, n_sms)) * 4);
     pl.xp = take((size_t)pl.max_rows * d * 2);
     pl.act = take((size_t)pl.max_rows * F * 2);
     pl.out = take((size_t)pl.max_rows * d * 4);
@@ -294,14 +296,20 @@ int xs::forward_impl(const FwdCall &c, FwdStep step) {
   };
   if (!mark(0)) return XS_ERR_CUDA;
   cudaError_t re;
+  int32_t *rstat = at<int32_t>(workspace, pl.rstat);
+  a.router_status = rstat;
   if (B >= kRouterTcMinB) {
-    int32_t *rstat = at<int32_t>(workspace, pl.rstat);
     int grid = 0;
     re = launch_router_tc(c.x, c.W_g, h, B, N, d, a.done, rstat, sms, &grid, s);
-    a.router_status = rstat;
     a.router_ctas = grid;
-  } else {
+  } else if (d < kRouterSplitMinD || d > kRouterSplitMaxD) {
     re = launch_router_logits(c.x, c.W_g, h, B, N, d, a.done, s);
+    a.router_status = nullptr;
+  } else {
+    const int S = router_split_count(B, N, d, sms);
+    re = launch_router_split(c.x, c.W_g, h, B, N, d, S, a.done, rstat, s);
+    a.h_splits = S;
+    a.router_ctas = router_split_ctas(B, N, d, sms);
   }
   if (re != cudaSuccess || !mark(1)) return XS_ERR_CUDA;
   a.events = events ? events + 2 : nullptr;  // between the selection and refinement kernels

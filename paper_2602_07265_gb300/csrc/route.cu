@@ -596,14 +596,25 @@ __device__ __forceinline__ void token_scores(const RouteArgs &a, int t, int lane
                                              bool write_p) {
   const int N = a.N;
   if (a.logits != nullptr) {
+    // The router may leave the logits as slices over d (h[s][t][j]); they
+    // are added in slice order.
     const float *hrow = a.logits + (size_t)t * N;
-    float mx = -INFINITY;
 #pragma unroll
     for (int q = 0; q < kQ; ++q) {
       const int j = lane + 32 * q;
       vals[q] = (j < N) ? hrow[j] : -INFINITY;
-      mx = fmaxf(mx, vals[q]);
     }
+    for (int sl = 1; sl < a.h_splits; ++sl) {
+      const float *hs = hrow + (size_t)sl * a.B * N;
+#pragma unroll
+      for (int q = 0; q < kQ; ++q) {
+        const int j = lane + 32 * q;
+        if (j < N) vals[q] = __fadd_rn(vals[q], hs[j]);
+      }
+    }
+    float mx = -INFINITY;
+#pragma unroll
+    for (int q = 0; q < kQ; ++q) mx = fmaxf(mx, vals[q]);
 #pragma unroll
     for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, o));
     float sum = 0.f;

@@ -99,6 +99,7 @@ Plan make_plan(int B, int N, int k, int d, int F, bool with_ffn, int n_sms, int 
 
 struct RouteArgs {
   const float *logits;   // nullable: if set, p = softmax(logits) is computed first
+  int h_splits;          // logits as h_splits slices [h_splits][B][N], added in slice order
   float *p;              // [B, N] scores (input if logits == nullptr, else output)
   int B, N, k, budget, mode, k0, m_r, T, G, m_g;
   float tau;             // THRESH: covered fraction of the score mass
@@ -132,8 +133,19 @@ struct RouteArgs {
 };
 
 cudaError_t launch_route(const RouteArgs &a, cudaStream_t s);
+// Router logits for B < kRouterTcMinB.  d outside [kRouterSplitMinD,
+// kRouterSplitMaxD]: whole-d blocks of 8 tokens x 4 experts (route.cu),
+// h[t][e].  d inside: d-sliced blocks (router_split.cu), h[s][t][e] for s <
+// router_split_count(), one slice of d each, which the selection kernel
+// adds in order; status: [router_split_ctas()] words, one per CTA.
+constexpr int kRouterSplitMinD = 4096;
+constexpr int kRouterSplitMaxD = 16384;
 cudaError_t launch_router_logits(const uint16_t *x, const float *Wg, float *h, int B, int N,
                                  int d, int32_t *done, cudaStream_t s);
+int router_split_count(int B, int N, int d, int n_sms);
+int router_split_ctas(int B, int N, int d, int n_sms);
+cudaError_t launch_router_split(const uint16_t *x, const float *Wg, float *h, int B, int N, int d,
+                                int S, int32_t *done, int32_t *status, cudaStream_t s);
 // The router on the tensor cores (router_tc.cu).  status: [router_tc_ctas()]
 // words, an upper bound on its grid; each launched CTA writes its word.
 constexpr int kRouterTcMinB = 64;   // batches from this size use it

@@ -335,11 +335,20 @@ def test_forward_shared_experts_full_size_sampled(X):
     assert not np.array_equal(g0["y"], g["y"])
 
 
-# ---- router logits on either path (CUDA cores below 64 tokens, tensor cores from 64) ----
+# ---- router logits on every path (CUDA cores below 64 tokens: whole-d blocks
+# below d = 4096, d-sliced blocks from it; tensor cores from 64 tokens) ----
 # Below 64 tokens: one or two token blocks, ragged expert blocks (N = 100),
 # every cluster split of d (d = 128: 1; 512: 4; 2048 and 7168: 8 or 4) and the
-# unsplit grid of N = 1024.
+# unsplit grid of N = 1024.  The d-sliced router: 1, 2 and 4 token groups per
+# lane (B = 1, 13, 37, 63), ragged expert blocks (N = 100, 250), ragged
+# slices (d = 4224 = 66 columns of 64), 1 to 128 expert blocks and 2, 4 and 8
+# slices (d = 16384).
 @pytest.mark.parametrize("w", [
+    W.TINY.with_(d=4096, F=128, B=1, budget=8), W.TINY.with_(N=100, d=4224, F=128, B=13),
+    W.TINY.with_(N=250, d=4096, F=128, B=37, budget=24),
+    W.TINY.with_(N=8, k=4, d=8192, F=128, B=63, budget=4),
+    W.TINY.with_(N=1024, k=16, d=4096, F=128, B=20, budget=64),
+    W.TINY.with_(N=32, d=16384, F=128, B=9, budget=8), W.DSR1.with_(B=8),
     W.TINY.with_(B=1, budget=8), W.TINY.with_(B=33), W.TINY.with_(N=100, B=40),
     W.TINY.with_(d=128, F=128, B=20, budget=8), W.TINY.with_(N=1024, k=16, budget=64, B=16),
     W.TINY.with_(B=63), W.TINY.with_(B=64), W.TINY.with_(B=65, budget=16),
