@@ -122,10 +122,13 @@ __device__ __forceinline__ int lane_take(LaneList<Q> &L, int count, Emit emit) {
 // lane list laid out by lane_load (lane l slot q: index j0 + l + 32 q), in
 // the order of `before`: every candidate whose key is above the count-th
 // largest key T, then the lowest-index candidates whose key equals T.  T is
-// found bit by bit from the top (the largest T with count(key >= T) >=
-// count), one warp reduction per bit; the search stops early once a
-// threshold has exactly `count` keys at or above it.  All of them if count
-// >= the live candidates.
+// the largest key with count(key >= T) >= count, found bit by bit from the
+// top: the bits above the highest bit where the largest and smallest live
+// keys differ are theirs, and the rest are found two bits per round (three
+// independent warp reductions).  The search stops early once a threshold has
+// exactly `count` keys at or above it (those are the count best: any such
+// threshold marks the same set).  All of them if count >= the live
+// candidates.
 template <int Q, class Mark>
 __device__ __forceinline__ void lane_mark_top(const LaneList<Q> &L, int count, Mark mark) {
   const int lane = threadIdx.x & 31;
@@ -140,21 +143,46 @@ __device__ __forceinline__ void lane_mark_top(const LaneList<Q> &L, int count, M
       if (L.key[q] != 0u) mark(L.idx[q]);
     return;
   }
-  uint32_t T = 0u;
-  for (int bit = 31; bit >= 0; --bit) {
-    const uint32_t c = T | (1u << bit);
+  uint32_t kmx = 0u, kmn = 0xffffffffu;
+#pragma unroll
+  for (int q = 0; q < Q; ++q)
+    if (L.key[q] != 0u) {
+      kmx = max(kmx, L.key[q]);
+      kmn = min(kmn, L.key[q]);
+    }
+  kmx = __reduce_max_sync(kFull, kmx);
+  kmn = __reduce_min_sync(kFull, kmn);
+  const uint32_t diff = kmx ^ kmn;
+  int bit = diff != 0u ? 31 - __clz(diff) : -1;
+  // The shared high bits (2u << 31 wraps to 0: nothing shared).
+  uint32_t T = diff != 0u ? (kmx & ~((2u << bit) - 1u)) : kmx;
+  // Exactly `count` keys are >= c and every other key is below c: they are
+  // the count best, whatever the order among them.
+  auto mark_from = [&](uint32_t c) {
+#pragma unroll
+    for (int q = 0; q < Q; ++q)
+      if (L.key[q] >= c) mark(L.idx[q]);
+  };
+  auto count_from = [&](uint32_t c) {
     int n = 0;
 #pragma unroll
     for (int q = 0; q < Q; ++q) n += L.key[q] >= c ? 1 : 0;
-    n = static_cast<int>(__reduce_add_sync(kFull, static_cast<unsigned>(n)));
-    if (n == count) {
-      // Exactly `count` keys are >= c and every other key is below c: they
-      // are the count best, whatever the order among them.
-#pragma unroll
-      for (int q = 0; q < Q; ++q)
-        if (L.key[q] >= c) mark(L.idx[q]);
-      return;
-    }
+    return n;
+  };
+  for (; bit >= 1; bit -= 2) {
+    const uint32_t c1 = T | (1u << (bit - 1)), c2 = T | (2u << (bit - 1)), c3 = T | (3u << (bit - 1));
+    const int n1 = static_cast<int>(__reduce_add_sync(kFull, static_cast<unsigned>(count_from(c1))));
+    const int n2 = static_cast<int>(__reduce_add_sync(kFull, static_cast<unsigned>(count_from(c2))));
+    const int n3 = static_cast<int>(__reduce_add_sync(kFull, static_cast<unsigned>(count_from(c3))));
+    if (n3 == count) return mark_from(c3);
+    if (n2 == count) return mark_from(c2);
+    if (n1 == count) return mark_from(c1);
+    T = n3 > count ? c3 : n2 > count ? c2 : n1 > count ? c1 : T;
+  }
+  if (bit == 0) {
+    const uint32_t c = T | 1u;
+    const int n = static_cast<int>(__reduce_add_sync(kFull, static_cast<unsigned>(count_from(c))));
+    if (n == count) return mark_from(c);
     if (n > count) T = c;
   }
   int gt = 0;
@@ -589,6 +617,132 @@ __device__ void build_permutation(const RouteArgs &a, PermSmem sm) {
   }
 }
 
+// The same permutation, tiles and statistics as build_permutation, for a
+// batch of at most 32 tokens whose ids are in shared memory (ids_s[t * k +
+// s]), with two block barriers instead of about ten.  A pair's position in
+// its expert's run is the number of earlier tokens routed to that expert (a
+// token uses an expert in at most one slot), so one 32-bit token mask per
+// expert gives the counts and every position.  The masks (sm.cursor, as
+// uint32) must be zero on entry.
+//   1. every pair (t, s): mask[e] |= 1 << t (shared-memory atomic).
+//   2. warp 0, 32 experts per round: counts, exclusive prefix over the
+//      experts (rows, and tiles = used experts: a count of at most 32 is one
+//      tile), tiles, meta.
+//   3. warp t, lane s < k: position of pair (t, s) = offset[e] +
+//      popc(mask[e] & (tokens below t)).
+__device__ void build_permutation_small(const RouteArgs &a, PermSmem sm, const int32_t *ids_s) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int nwarps = blockDim.x >> 5;
+  const int B = a.B, N = a.N, k = a.k;
+  uint32_t *s_tmask = reinterpret_cast<uint32_t *>(sm.cursor);  // [N] token mask per expert
+  int32_t *s_off = sm.chunk;                                     // [N] first row per expert
+  for (int q = tid; q < B * k; q += blockDim.x) {
+    const int e = ids_s[q];
+    if ((unsigned)e < (unsigned)N) atomicOr(&s_tmask[e], 1u << (q / k));
+  }
+  __syncthreads();
+  if (warp == 0) {
+    const int G = a.ep_ranks > 1 ? a.ep_ranks : 1, g = G > 1 ? a.ep_rank : 0;
+    const int e_lo = g * (N / G), e_hi = (g + 1) * (N / G);
+    Meta *m = a.meta;
+    int rows0 = 0, tiles0 = 0;  // totals of the rounds before
+    for (int e0 = 0; e0 < N; e0 += 32) {
+      const int e = e0 + lane;
+      const int c = e < N ? __popc(s_tmask[e]) : 0;
+      const int u = c > 0 ? 1 : 0;
+      int rx = c, ux = u;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int r1 = __shfl_up_sync(kFull, rx, o), u1 = __shfl_up_sync(kFull, ux, o);
+        if (lane >= o) {
+          rx += r1;
+          ux += u1;
+        }
+      }
+      const int row = rows0 + rx - c, tile = tiles0 + ux - u;  // exclusive
+      if (e < N) {
+        s_off[e] = row;
+        a.counts[e] = c;
+        a.offsets[e] = row;
+        if (a.counts_out) a.counts_out[e] = c;
+        if (a.offsets_out) a.offsets_out[e] = row;
+        // This call's FFN work (Sec. 5): the tiles and rows of expert group
+        // ep_rank (a contiguous index range); without expert parallelism, all.
+        if (e == e_lo) {
+          m->ffn_t0 = tile;
+          m->row0 = row;
+        }
+        if (e_hi < N && e == e_hi) {
+          m->ffn_t1 = tile;
+          m->row1 = row;
+        }
+        if (c > 0) {
+          Tile tl;
+          tl.expert = e;
+          tl.row0 = row;
+          tl.ntok = c;
+          tl.pad = 0;
+          a.tiles[tile] = tl;
+        }
+      }
+      rows0 += __shfl_sync(kFull, rx, 31);
+      tiles0 += __shfl_sync(kFull, ux, 31);
+    }
+    const int tot_rows = rows0, tot_tiles = tiles0;
+    // Shared experts: every token, in token order, after the routed pairs
+    // (one tile each: B <= 32).
+    for (int j = lane; j < a.n_shared; j += 32) {
+      Tile tl;
+      tl.expert = N + j;
+      tl.row0 = tot_rows + j * B;
+      tl.ntok = B;
+      tl.pad = 0;
+      a.tiles[tot_tiles + j] = tl;
+    }
+    if (lane == 0) {
+      a.offsets[N] = tot_rows;
+      if (a.offsets_out) a.offsets_out[N] = tot_rows;
+      if (e_hi >= N) {
+        m->ffn_t1 = tot_tiles;
+        m->row1 = tot_rows;
+      }
+      const int own_shared = g == 0 ? 1 : 0;
+      m->ffn_s0 = tot_tiles;
+      m->ffn_s1 = tot_tiles + own_shared * a.n_shared;
+      m->srows = own_shared;
+      // Field by field: union_topk belongs to the union CTAs (score_kernel).
+      m->n_pairs = tot_rows;  // == B * kp unless scores were non-finite
+      m->n_tiles = tot_tiles + a.n_shared;
+      m->n_used = tot_tiles;
+      m->n_rows = tot_rows + a.n_shared * B;
+      if (a.stats) {
+        xs_stats *st = a.stats;
+        st->n_selected = m->n_selected;
+        st->n_used = tot_tiles;
+        st->max_group_load = m->max_group_load;
+        st->n_pairs = tot_rows;
+        st->status = m->status;
+        st->reserved[0] = st->reserved[1] = 0;
+      }
+    }
+  }
+  __syncthreads();
+  for (int t = warp; t < B; t += nwarps) {
+    if (lane < k) {
+      const int q = t * k + lane;
+      const int e = ids_s[q];
+      if ((unsigned)e < (unsigned)N) {
+        const int r = s_off[e] + __popc(s_tmask[e] & ((1u << t) - 1u));
+        a.perm[r] = q;
+        a.pos[q] = r;
+        if (a.perm_out) a.perm_out[r] = q;
+      } else {
+        a.pos[q] = -1;
+      }
+    }
+  }
+}
+
 // Token t's dense scores (a2) in vals[q] = p[t, lane + 32 q] (0 past N): the
 // softmax of its logits (written to a.p when write_p), or the given scores.
 template <int kQ>
@@ -704,6 +858,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   __shared__ int32_t s_cursor[kMaxN];
   __shared__ int32_t s_chunk[kMaxN];
   __shared__ int32_t s_tmp[200];
+  __shared__ int s_rflag;               // a router CTA reported a timeout
 
   pdl_wait();
   pdl_trigger();
@@ -711,6 +866,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   const int nwarps = blockDim.x >> 5;
   const int B = a.B, N = a.N, k = a.k;
   const int C = chunk_count(B), c = blockIdx.x;
+  if (tid == 0) s_rflag = 0;
   if (c >= C) {  // CTAs C .. 2C - 1 count the plain top-k union
     union_cta<kQ>(a, s_union, s_scal);
     return;
@@ -980,13 +1136,26 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   }
   __syncthreads();
 
+  // The router's status (if it reports one) rides on the barrier of the
+  // selection statistics through a shared flag.  The token masks of the
+  // small-batch permutation are cleared before that barrier too.
+  if (C == 1)
+    for (int j = tid; j < N; j += blockDim.x) s_cursor[j] = 0;
   int nsel, maxload;
-  if (tid == 0) s_gl[kMaxN] = 0;
-  selection_stats(a, s_mask, s_gl, nsel, maxload);
+  {
+    int rs = 0;
+    for (int i = tid; i < a.router_ctas; i += blockDim.x) rs |= __ldcg(a.router_status + i);
+    if (rs != 0) s_rflag = 1;
+  }
+  if (a.G <= 1) {  // one group: its load is |S|
+    nsel = __syncthreads_count(tid < N && s_mask[tid]);
+    maxload = nsel;
+  } else {
+    if (tid == 0) s_gl[kMaxN] = 0;
+    selection_stats(a, s_mask, s_gl, nsel, maxload);
+  }
+  const int rstat = s_rflag;
   for (int j = tid; j < N; j += blockDim.x) a.mask[j] = s_mask[j];
-  int rstat = 0;  // the router's status, if it reports one
-  for (int i = tid; i < a.router_ctas; i += blockDim.x) rstat = max(rstat, __ldcg(a.router_status + i));
-  rstat = __syncthreads_or(rstat);
   if (tid == 0) {
     // Field by field: union_topk belongs to the union CTAs.
     Meta *m = a.meta;
@@ -1001,8 +1170,9 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   }
   if (!a.fuse_refine) return;
   // Small batches: refinement and permutation in this CTA too (no second
-  // kernel); this chunk's scores are still in shared memory.
-  __syncthreads();
+  // kernel); this chunk's scores are still in shared memory.  (The mask is
+  // complete since the statistics' barrier; nothing the refinement writes
+  // is read before it.)
   int32_t *ids_s = C == 1 ? &s_top[0][0] : nullptr;  // one chunk: ids stay in shared memory
   refine_tokens<kQ>(
       a, s_mask, nsel, s_chunk, s_tmp, 0, B, min(k, nsel),
@@ -1013,8 +1183,12 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
       ids_s);
   if (C > 1) __threadfence();
   __syncthreads();
-  build_permutation(a, PermSmem{s_counts, s_cursor, s_chunk, s_tmp, s_scal,
-                                reinterpret_cast<int32_t *>(ps + kChunk * N), ids_s});
+  if (C == 1)
+    build_permutation_small(a, PermSmem{s_counts, s_cursor, s_chunk, s_tmp, s_scal, nullptr, nullptr},
+                            ids_s);
+  else
+    build_permutation(a, PermSmem{s_counts, s_cursor, s_chunk, s_tmp, s_scal,
+                                  reinterpret_cast<int32_t *>(ps + kChunk * N), ids_s});
 }
 
 template <int kQ>
