@@ -618,27 +618,31 @@ __device__ void build_permutation(const RouteArgs &a, PermSmem sm) {
 }
 
 // The same permutation, tiles and statistics as build_permutation, for a
-// batch of at most 32 tokens whose ids are in shared memory (ids_s[t * k +
-// s]), with two block barriers instead of about ten.  A pair's position in
-// its expert's run is the number of earlier tokens routed to that expert (a
-// token uses an expert in at most one slot), so one 32-bit token mask per
-// expert gives the counts and every position.  The masks (sm.cursor, as
-// uint32) must be zero on entry.
-//   1. every pair (t, s): mask[e] |= 1 << t (shared-memory atomic).
+// batch of at most 64 tokens, with two block barriers instead of about ten.
+// A pair's position in its expert's run is the number of earlier tokens
+// routed to that expert (a token uses an expert in at most one slot), so one
+// 32-bit token mask per expert and 32-token chunk gives the counts and every
+// position.  The masks (sm.cursor for tokens 0-31, sm.counts for 32-63, as
+// uint32) must be zero on entry.  ids: ids_s[t * k + s] in shared memory
+// (one chunk), else the ids in global memory.
+//   1. every pair (t, s): mask[t / 32][e] |= 1 << (t % 32) (shared-memory
+//      atomic).
 //   2. warp 0, 32 experts per round: counts, exclusive prefix over the
-//      experts (rows, and tiles = used experts: a count of at most 32 is one
+//      experts (rows, and tiles = used experts: a count of at most 64 is one
 //      tile), tiles, meta.
-//   3. warp t, lane s < k: position of pair (t, s) = offset[e] +
-//      popc(mask[e] & (tokens below t)).
+//   3. warp t, lane s < k: position of pair (t, s) = offset[e] + the tokens
+//      of e in the chunks before + popc(mask[t / 32][e] & (tokens below t)).
 __device__ void build_permutation_small(const RouteArgs &a, PermSmem sm, const int32_t *ids_s) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nwarps = blockDim.x >> 5;
   const int B = a.B, N = a.N, k = a.k;
-  uint32_t *s_tmask = reinterpret_cast<uint32_t *>(sm.cursor);  // [N] token mask per expert
-  int32_t *s_off = sm.chunk;                                     // [N] first row per expert
+  uint32_t *s_tm0 = reinterpret_cast<uint32_t *>(sm.cursor);  // [N] tokens 0-31 per expert
+  uint32_t *s_tm1 = reinterpret_cast<uint32_t *>(sm.counts);  // [N] tokens 32-63 per expert
+  int32_t *s_off = sm.chunk;                                   // [N] first row per expert
+  auto id_of = [&](int q) { return ids_s != nullptr ? ids_s[q] : __ldcg(a.ids + q); };
   for (int q = tid; q < B * k; q += blockDim.x) {
-    const int e = ids_s[q];
-    if ((unsigned)e < (unsigned)N) atomicOr(&s_tmask[e], 1u << (q / k));
+    const int e = id_of(q), t = q / k;
+    if ((unsigned)e < (unsigned)N) atomicOr(t < 32 ? &s_tm0[e] : &s_tm1[e], 1u << (t & 31));
   }
   __syncthreads();
   if (warp == 0) {
@@ -648,7 +652,7 @@ __device__ void build_permutation_small(const RouteArgs &a, PermSmem sm, const i
     int rows0 = 0, tiles0 = 0;  // totals of the rounds before
     for (int e0 = 0; e0 < N; e0 += 32) {
       const int e = e0 + lane;
-      const int c = e < N ? __popc(s_tmask[e]) : 0;
+      const int c = e < N ? __popc(s_tm0[e]) + (B > 32 ? __popc(s_tm1[e]) : 0) : 0;
       const int u = c > 0 ? 1 : 0;
       int rx = c, ux = u;
 #pragma unroll
@@ -690,7 +694,7 @@ __device__ void build_permutation_small(const RouteArgs &a, PermSmem sm, const i
     }
     const int tot_rows = rows0, tot_tiles = tiles0;
     // Shared experts: every token, in token order, after the routed pairs
-    // (one tile each: B <= 32).
+    // (one tile each: B <= 64).
     for (int j = lane; j < a.n_shared; j += 32) {
       Tile tl;
       tl.expert = N + j;
@@ -730,9 +734,11 @@ __device__ void build_permutation_small(const RouteArgs &a, PermSmem sm, const i
   for (int t = warp; t < B; t += nwarps) {
     if (lane < k) {
       const int q = t * k + lane;
-      const int e = ids_s[q];
+      const int e = id_of(q);
       if ((unsigned)e < (unsigned)N) {
-        const int r = s_off[e] + __popc(s_tmask[e] & ((1u << t) - 1u));
+        const uint32_t below = (1u << (t & 31)) - 1u;
+        const int r = s_off[e] + (t < 32 ? __popc(s_tm0[e] & below)
+                                         : __popc(s_tm0[e]) + __popc(s_tm1[e] & below));
         a.perm[r] = q;
         a.pos[q] = r;
         if (a.perm_out) a.perm_out[r] = q;
@@ -1139,8 +1145,11 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   // The router's status (if it reports one) rides on the barrier of the
   // selection statistics through a shared flag.  The token masks of the
   // small-batch permutation are cleared before that barrier too.
-  if (C == 1)
-    for (int j = tid; j < N; j += blockDim.x) s_cursor[j] = 0;
+  if (C <= 2)
+    for (int j = tid; j < N; j += blockDim.x) {
+      s_cursor[j] = 0;
+      s_counts[j] = 0;
+    }
   int nsel, maxload;
   {
     int rs = 0;
@@ -1183,12 +1192,9 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
       ids_s);
   if (C > 1) __threadfence();
   __syncthreads();
-  if (C == 1)
-    build_permutation_small(a, PermSmem{s_counts, s_cursor, s_chunk, s_tmp, s_scal, nullptr, nullptr},
-                            ids_s);
-  else
-    build_permutation(a, PermSmem{s_counts, s_cursor, s_chunk, s_tmp, s_scal,
-                                  reinterpret_cast<int32_t *>(ps + kChunk * N), ids_s});
+  static_assert(kFuseChunks <= 2, "the fused permutation takes at most two 32-token chunks");
+  build_permutation_small(a, PermSmem{s_counts, s_cursor, s_chunk, s_tmp, s_scal, nullptr, nullptr},
+                          ids_s);
 }
 
 template <int kQ>
