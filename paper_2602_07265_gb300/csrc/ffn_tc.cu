@@ -235,18 +235,50 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
   };
   const bool producer = warp == 0 && lane == 0;
   const int n_pre = (it_end - it_begin) < C::kStages ? static_cast<int>(it_end - it_begin) : C::kStages;
-  // The producer walks its K steps with a cursor (unit u, step kk of it) and
-  // re-reads the unit's source only when u changes.
-  struct Cursor {
+  // The CTA's steps as segments (unit u, steps [k0, k1) of it), in the order
+  // all three roles process them: first the piece of the last unit that the
+  // next CTA finishes, then the piece of the first unit that the previous
+  // CTA began, then the whole units between.  Both pieces of every unit cut
+  // between two CTAs are then done early, so their partial sums are added
+  // early too, and a CTA ends on a whole unit (whose epilogue is one TMEM
+  // drain) instead of a cut one (partial store, fence, arrival, the other
+  // pieces' loads).  Results do not depend on the order: the pieces are
+  // added in CTA order.
+  struct Seg {
     long long u;
-    int kk;
+    int k0, k1;
+  };
+  const long long u_first = it_begin / KI, u_last = (it_end - 1) / KI;
+  const int kT0 = static_cast<int>(it_begin - u_first * KI);  // the first unit starts here
+  const int kH1 = static_cast<int>(it_end - u_last * KI);     // the last unit ends here
+  const bool one_unit = u_first == u_last;
+  const int nH = (!one_unit && kH1 < KI) ? 1 : 0, nT = (!one_unit && kT0 > 0) ? 1 : 0;
+  const long long fu0 = u_first + nT;                          // first whole unit
+  const int n_seg = one_unit ? 1 : nH + nT + static_cast<int>(u_last - nH - fu0 + 1);
+  auto seg_at = [&](int i) -> Seg {
+    if (one_unit) return Seg{u_first, kT0, kH1};
+    if (i < nH) return Seg{u_last, 0, kH1};
+    if (i < nH + nT) return Seg{u_first, kT0, KI};
+    return Seg{fu0 + (i - nH - nT), 0, KI};
+  };
+  // The producer walks its K steps with a cursor (segment si: unit u, step
+  // kk of [.., k1)) and re-reads the unit's source only when u changes.
+  struct Cursor {
+    int si;
+    long long u;
+    int kk, k1;
     bool fresh;
   };
-  const Cursor c_begin{it_begin / KI, static_cast<int>(it_begin % KI), true};
+  const Seg s0 = seg_at(0);
+  const Cursor c_begin{0, s0.u, s0.k0, s0.k1, true};
   auto advance = [&](Cursor &c) {
-    if (++c.kk == KI) {
-      c.kk = 0;
-      ++c.u;
+    if (++c.kk == c.k1) {
+      if (++c.si < n_seg) {
+        const Seg g = seg_at(c.si);
+        c.u = g.u;
+        c.kk = g.k0;
+        c.k1 = g.k1;
+      }
       c.fresh = true;
     }
   };
@@ -331,10 +363,10 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
       uint32_t phase = 0;
       int segi = 0;
       bool ok = true, any = false;
-      for (long long it = it_begin; ok && it < it_end; ++segi) {
-        const long long u = it / KI;
-        const int k0 = static_cast<int>(it - u * KI);
-        const int k1 = static_cast<int>(k0 + (it_end - it) < KI ? k0 + (it_end - it) : KI);
+      for (; ok && segi < n_seg; ++segi) {
+        const Seg g = seg_at(segi);
+        const long long u = g.u;
+        const int k0 = g.k0, k1 = g.k1;
         const Tile tl = p.tiles[wt.tile(static_cast<int>(u / MT))];
         const int n_mma = ((tl.ntok + 15) / 16) * 16;
         const uint32_t idesc = idesc_bf16(kBM, n_mma);
@@ -370,7 +402,6 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
         }
         if (!ok) break;
         mma_commit(accfull_bar(buf));
-        it += k1 - k0;
       }
       if (!ok) {
         set_status(p, XS_DEV_TIMEOUT);
@@ -387,11 +418,10 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
     const int q = warp & 3;                  // TMEM lane quarter of this warp
     const int row = q * 32 + lane;           // weight row inside the unit
     const bool leader = threadIdx.x == 64;
-    int segi = 0;
-    for (long long it = it_begin; it < it_end; ++segi) {
-      const long long u = it / KI;
-      const int k0 = static_cast<int>(it - u * KI);
-      const int k1 = static_cast<int>(k0 + (it_end - it) < KI ? k0 + (it_end - it) : KI);
+    for (int segi = 0; segi < n_seg; ++segi) {
+      const Seg g = seg_at(segi);
+      const long long u = g.u;
+      const int k0 = g.k0, k1 = g.k1;
       const Tile tl = p.tiles[wt.tile(static_cast<int>(u / MT))];
       const int mt = static_cast<int>(u % MT);
       const int n_mma = ((tl.ntok + 15) / 16) * 16;
@@ -449,10 +479,15 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
             if (kGateUp) mine[(128 + c0 + j) * 128 + row] = v[j];
           }
         }
+        // The accumulator is free once the sums are in the partial buffer:
+        // the MMAs of the next segment go on while this piece arrives and,
+        // if it is the last, adds the pieces (from the buffers) and emits.
         __threadfence();
+        tc_fence_before();
         named_bar_sync(1, kEpiThreads);
         const int c_first = rg.cta_of(u * KI), c_last = rg.cta_of(u * KI + KI - 1);
         if (leader) {
+          mbar_arrive(accempty_bar(buf));
           const int old = atomicAdd(&p.cnt[u], 1);
           *s_flag = (old == c_last - c_first) ? 1 : 0;
         }
@@ -480,11 +515,11 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
             emit(c0, g, v);
           }
         }
+        continue;  // accumulator released above
       }
       tc_fence_before();
       named_bar_sync(1, kEpiThreads);
       if (leader) mbar_arrive(accempty_bar(buf));
-      it += k1 - k0;
     }
   }
 
