@@ -466,56 +466,88 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
           emit(c0, g, v);
         }
       } else {
-        // Piece of a unit shared with other CTAs: publish the partial sums.
-        const int my_slot = rg.slot(cta, u);
-        float *mine = p.part + static_cast<size_t>(cta * 2 + my_slot) * C::kNumA * 128 * 128;
-        for (int c0 = 0; c0 < n_mma; c0 += 16) {
-          float g[16], v[16];
-          tmem_ld16(tacc + c0, g);
-          if (kGateUp) tmem_ld16(tacc + 128 + c0, v);
-#pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            mine[(c0 + j) * 128 + row] = g[j];
-            if (kGateUp) mine[(128 + c0 + j) * 128 + row] = v[j];
-          }
-        }
-        // The accumulator is free once the sums are in the partial buffer:
-        // the MMAs of the next segment go on while this piece arrives and,
-        // if it is the last, adds the pieces (from the buffers) and emits.
-        __threadfence();
-        tc_fence_before();
-        named_bar_sync(1, kEpiThreads);
         const int c_first = rg.cta_of(u * KI), c_last = rg.cta_of(u * KI + KI - 1);
-        if (leader) {
-          mbar_arrive(accempty_bar(buf));
-          const int old = atomicAdd(&p.cnt[u], 1);
-          *s_flag = (old == c_last - c_first) ? 1 : 0;
-        }
+        // Piece of a unit shared with other CTAs.  If every other piece has
+        // already arrived (its sums are in its partial buffer), this one is
+        // the last: it adds them to its own sums straight from TMEM, in CTA
+        // order as below (same bits), without storing, fencing or arriving.
+        if (leader) *s_flag = ld_acquire_gpu(p.cnt + u) == c_last - c_first ? 1 : 0;
         named_bar_sync(1, kEpiThreads);
-        const bool last = *s_flag != 0;
+        const bool direct_last = *s_flag != 0;
         named_bar_sync(1, kEpiThreads);
-        if (last) {
+        if (direct_last) {
           __threadfence();
           for (int c0 = 0; c0 < n_mma; c0 += 16) {
-            float g[16], v[16];
+            float og[16], ov[16], g[16], v[16];
+            tmem_ld16(tacc + c0, og);
+            if (kGateUp) tmem_ld16(tacc + 128 + c0, ov);
 #pragma unroll
             for (int j = 0; j < 16; ++j) g[j] = v[j] = 0.f;
             for (int c = c_first; c <= c_last; ++c) {
               const float *src = p.part + static_cast<size_t>(c * 2 + rg.slot(c, u)) * C::kNumA * 128 * 128;
 #pragma unroll
               for (int j = 0; j < 16; ++j) {
-                const float a = __ldcg(src + (c0 + j) * 128 + row);
+                const float a = c == cta ? og[j] : __ldcg(src + (c0 + j) * 128 + row);
                 g[j] = (c == c_first) ? a : g[j] + a;
                 if (kGateUp) {
-                  const float b = __ldcg(src + (128 + c0 + j) * 128 + row);
+                  const float b = c == cta ? ov[j] : __ldcg(src + (128 + c0 + j) * 128 + row);
                   v[j] = (c == c_first) ? b : v[j] + b;
                 }
               }
             }
             emit(c0, g, v);
           }
+        } else {
+          // Publish the partial sums.
+          const int my_slot = rg.slot(cta, u);
+          float *mine = p.part + static_cast<size_t>(cta * 2 + my_slot) * C::kNumA * 128 * 128;
+          for (int c0 = 0; c0 < n_mma; c0 += 16) {
+            float g[16], v[16];
+            tmem_ld16(tacc + c0, g);
+            if (kGateUp) tmem_ld16(tacc + 128 + c0, v);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              mine[(c0 + j) * 128 + row] = g[j];
+              if (kGateUp) mine[(128 + c0 + j) * 128 + row] = v[j];
+            }
+          }
+          // The accumulator is free once the sums are in the partial buffer:
+          // the MMAs of the next segment go on while this piece arrives and,
+          // if it is the last, adds the pieces (from the buffers) and emits.
+          __threadfence();
+          tc_fence_before();
+          named_bar_sync(1, kEpiThreads);
+          if (leader) {
+            mbar_arrive(accempty_bar(buf));
+            const int old = atomicAdd(&p.cnt[u], 1);
+            *s_flag = (old == c_last - c_first) ? 1 : 0;
+          }
+          named_bar_sync(1, kEpiThreads);
+          const bool last = *s_flag != 0;
+          named_bar_sync(1, kEpiThreads);
+          if (last) {
+            __threadfence();
+            for (int c0 = 0; c0 < n_mma; c0 += 16) {
+              float g[16], v[16];
+#pragma unroll
+              for (int j = 0; j < 16; ++j) g[j] = v[j] = 0.f;
+              for (int c = c_first; c <= c_last; ++c) {
+                const float *src = p.part + static_cast<size_t>(c * 2 + rg.slot(c, u)) * C::kNumA * 128 * 128;
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                  const float a = __ldcg(src + (c0 + j) * 128 + row);
+                  g[j] = (c == c_first) ? a : g[j] + a;
+                  if (kGateUp) {
+                    const float b = __ldcg(src + (128 + c0 + j) * 128 + row);
+                    v[j] = (c == c_first) ? b : v[j] + b;
+                  }
+                }
+              }
+              emit(c0, g, v);
+            }
+          }
+          continue;  // accumulator released above
         }
-        continue;  // accumulator released above
       }
       tc_fence_before();
       named_bar_sync(1, kEpiThreads);

@@ -113,6 +113,14 @@ __device__ __forceinline__ void bulk_prefetch_l2(const void *src, uint32_t bytes
                : "memory");
 }
 
+// ---------------------------------------------------------------- flags
+
+__device__ __forceinline__ int ld_acquire_gpu(const int32_t *p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
 // ---------------------------------------------------------------- tcgen05
 
 __device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
