@@ -283,6 +283,29 @@ def test_forward_expert_with_many_tokens(X):
     compare(w, g, x, W_g, weights, tokens=[0, 5, 100, 511])
 
 
+@pytest.mark.parametrize("w", [
+    # 2 used experts x 1 row block x 112 K steps over 28 CTAs of 8 steps: every
+    # gate/up unit is cut into 14 pieces (a CTA's range lies inside one unit).
+    W.TINY.with_(N=8, k=2, d=7168, F=128, B=5, budget=2, k0=0),
+    # 3 used experts: gate/up units of 112 steps cut into about 4 pieces,
+    # down units of 32 steps into 2.
+    W.TINY.with_(N=8, k=2, d=7168, F=2048, B=7, budget=3, k0=0),
+], ids=["units-cut-14-ways", "units-cut-2-to-4-ways"])
+def test_forward_units_cut_across_ctas(X, w):
+    """FFN units whose K steps are spread over many CTAs: each CTA does the
+    pieces it shares with its neighbours first, the last piece to arrive adds
+    them all (in CTA order).  Every token against the oracle; the packed path
+    gives the same bits, and so does a second call."""
+    x, W_g = W.router_inputs(w, 4)
+    weights = device_weights(w, 4)
+    g = gpu_forward(X, w, x, W_g, weights)
+    compare(w, g, x, W_g, weights)
+    g2 = gpu_forward_packed(X, w, x, W_g, weights)
+    assert np.array_equal(g["y"], g2["y"])
+    g3 = gpu_forward(X, w, x, W_g, weights)
+    assert np.array_equal(g["y"], g3["y"])
+
+
 def test_forward_deterministic(X):
     w = W.OLMOE.with_(B=32, budget=24, k0=1)
     x, W_g = W.router_inputs(w, 0)
