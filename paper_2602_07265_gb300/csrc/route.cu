@@ -953,7 +953,11 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   __syncthreads();
 
   // ---- the chunk's column-sum tree (a4) ----
+  // One chunk and no per-request step: the base set is final already, so
+  // the selection's mask starts from it here and two barriers are saved.
+  const bool one_pass = C == 1 && !hier;
   for (int j = tid; j < N; j += blockDim.x) {
+    if (one_pass) s_mask[j] = s_base[j];
     float v[kChunk];
 #pragma unroll
     for (int l = 0; l < kChunk; ++l) v[l] = ps[l * N + j];
@@ -1023,7 +1027,7 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
       s_base[j] = b;
     }
   }
-  __syncthreads();
+  if (!one_pass) __syncthreads();
 
   if (hier && !hier_here) {
     // Requests cross chunk boundaries: Algorithm 3 from the full score matrix.
@@ -1059,8 +1063,10 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
   }
 
   // ---- budgeted selection (a5) ----
-  for (int j = tid; j < N; j += blockDim.x) s_mask[j] = s_base[j];
-  __syncthreads();
+  if (!one_pass) {
+    for (int j = tid; j < N; j += blockDim.x) s_mask[j] = s_base[j];
+    __syncthreads();
+  }
   if (a.mode == XS_MODE_TOPK) {
     for (int j = tid; j < N; j += blockDim.x) s_mask[j] = 1;
   } else if (a.mode == XS_MODE_GROUP) {
