@@ -314,8 +314,23 @@ int xs::forward_impl(const FwdCall &c, FwdStep step) {
   if (re != cudaSuccess || !mark(1)) return XS_ERR_CUDA;
   a.events = events ? events + 2 : nullptr;  // between the selection and refinement kernels
   if (launch_route(a, s) != cudaSuccess || !mark(3)) return XS_ERR_CUDA;
+  // The gather kernel warms L2 with the gate/up kernel's first weights once
+  // the selected set is known (packed weights, without expert parallelism).
+  GatherPf pf;
+  std::memset(&pf, 0, sizeof(pf));
+  if (packed && !ep) {
+    pf.ready = a.done + 3;
+    pf.mask = a.mask;
+    pf.pk = static_cast<const uint8_t *>(c.P_gate_up);
+    pf.N = N;
+    pf.MT = F / 128;
+    pf.KI = d / 64;
+    pf.stage_bytes = 2 * 128 * 64 * 2;
+    pf.grid = sms;
+    pf.pf_bytes = kGatherPrefetchBytes;
+  }
   if (launch_gather(c.x, a.perm, a.meta, const_cast<uint16_t *>(f.xp), ep ? f.out : nullptr,
-                    pl.max_rows, B, d, k, s) != cudaSuccess ||
+                    pl.max_rows, B, d, k, pf, s) != cudaSuccess ||
       !mark(4))
     return XS_ERR_CUDA;
   if (launch_ffn_gate_up(f, s) != cudaSuccess || !mark(5)) return XS_ERR_CUDA;

@@ -17,6 +17,12 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 
+__device__ __forceinline__ unsigned long long gtimer() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
 // Order-preserving 32-bit key of an fp32 score (larger score -> larger key;
 // -0 is read as +0 so that equal scores get equal keys).  Key 0 marks "no
 // candidate": no finite score maps to it.
@@ -1170,7 +1176,16 @@ __global__ void __launch_bounds__(kRouteThreads, 1) score_kernel(RouteArgs a) {
     selection_stats(a, s_mask, s_gl, nsel, maxload);
   }
   const int rstat = s_rflag;
-  for (int j = tid; j < N; j += blockDim.x) a.mask[j] = s_mask[j];
+  // The mask, written by warp 0, then flagged (done[3]): the gather kernel,
+  // resident already, warms L2 with the weights the gate/up kernel will
+  // stream first while the refinement and permutation run.  The flag is a
+  // hint, not a release: a reader that sees it before the mask only
+  // prefetches other weights, so no fence slows this warp.
+  if (warp == 0) {
+    for (int j = lane; j < N; j += 32) a.mask[j] = s_mask[j];
+    __syncwarp();
+    if (lane == 0) *reinterpret_cast<volatile int32_t *>(a.done + 3) = 1;
+  }
   if (tid == 0) {
     // Field by field: union_topk belongs to the union CTAs.
     Meta *m = a.meta;
@@ -1267,7 +1282,7 @@ __global__ void __launch_bounds__(kRtWarps * 32) router_logits_kernel(
   __shared__ float red[kRtWarps][kRtOut];
   pdl_wait();
   pdl_trigger();
-  if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x < 3) done[threadIdx.x] = 0;
+  if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x < 4) done[threadIdx.x] = 0;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int e0 = blockIdx.x * kRtExp, t0 = blockIdx.y * kRtTok;
   const int d4 = d / 4;
@@ -1332,15 +1347,99 @@ __global__ void __launch_bounds__(kRtWarps * 32) router_logits_kernel(
   }
 }
 
+// L2 warm-up for the gate/up kernel (packed weights).  Its stream-K split
+// and segment order are those of ffn_tc.cu, predicted from the selected set
+// (one tile per selected expert, in expert order): CTA c of G takes steps
+// [I c / G, I (c + 1) / G) of I = |S| x MT x KI and does first the steps of
+// its last unit (if that unit continues in CTA c + 1), then those of its
+// first unit (if it began in CTA c - 1), then its whole units.  The first
+// pf_bytes of that order are prefetched into L2, by the first
+// kGatherWarmBlocks blocks (a few gate/up CTAs' ranges each: fewer blocks
+// waiting on the flag and a less bursty stream of prefetches measured
+// faster than one block per gate/up CTA).  A wrong prediction (an expert of
+// S with no token, or more than one tile) only prefetches other weights.
+__device__ void warm_gate_up(const GatherPf &g, int32_t *s_sel, int *s_n) {
+  const int tid = threadIdx.x, lane = tid & 31;
+  if (tid == 0) *s_n = -1;
+  __syncthreads();
+  if (tid < 32) {
+    // Wait (bounded: 2 ms, a hint only) for the selection kernel's mask.
+    bool ok = false;
+    if (lane == 0) {
+      const volatile int32_t *flag = g.ready;
+      ok = *flag != 0;
+      if (!ok) {
+        const unsigned long long t0 = gtimer();
+        while (!ok && gtimer() - t0 < 2000000ull) {
+          __nanosleep(256);
+          ok = *flag != 0;
+        }
+      }
+    }
+    ok = __shfl_sync(kFull, ok ? 1 : 0, 0) != 0;
+    if (ok) {
+      int n = 0;
+      for (int j0 = 0; j0 < g.N; j0 += 32) {
+        const bool sel = j0 + lane < g.N && __ldcg(g.mask + j0 + lane) != 0;
+        const unsigned b = __ballot_sync(kFull, sel);
+        if (sel) s_sel[n + __popc(b & ((1u << lane) - 1u))] = j0 + lane;
+        n += __popc(b);
+      }
+      if (lane == 0) *s_n = n;
+    }
+  }
+  __syncthreads();
+  const int nS = *s_n;
+  if (nS <= 0) return;
+  const long long KI = g.KI, I = static_cast<long long>(nS) * g.MT * KI;
+  const long long want = (I + 7) / 8;  // the FFN kernel's minimum of 8 steps per CTA
+  const int G = static_cast<int>(want < g.grid ? want : g.grid);
+  const int n_steps = g.pf_bytes / g.stage_bytes;
+  const int nb = gridDim.x < kGatherWarmBlocks ? static_cast<int>(gridDim.x) : kGatherWarmBlocks;
+  for (int c = blockIdx.x; c < G; c += nb) {
+    const long long ib = I * c / G, ie = I * (c + 1) / G;
+    const long long uf = ib / KI, ul = (ie - 1) / KI;
+    const long long kT0 = ib - uf * KI, kH1 = ie - ul * KI;
+    // The i-th step of the CTA's order, for i < n_steps (thread i issues it).
+    for (int i = tid; i < n_steps && i < ie - ib; i += blockDim.x) {
+      long long st;
+      if (uf == ul) {
+        st = ib + i;
+      } else {
+        const long long nH = kH1 < KI ? kH1 : 0, nT = kT0 > 0 ? KI - kT0 : 0;
+        if (i < nH)
+          st = ul * KI + i;
+        else if (i < nH + nT)
+          st = ib + (i - nH);
+        else
+          st = (uf + (kT0 > 0 ? 1 : 0)) * KI + (i - nH - nT);
+      }
+      const long long u = st / KI;
+      const int kk = static_cast<int>(st - u * KI);
+      const int e = s_sel[u / g.MT], mt = static_cast<int>(u % g.MT);
+      const uint8_t *blk =
+          g.pk + ((static_cast<size_t>(e) * g.MT + mt) * g.KI + kk) * static_cast<size_t>(g.stage_bytes);
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(blk)),
+                   "r"(g.stage_bytes)
+                   : "memory");
+    }
+  }
+}
+
 // Xp[row] = x[token of pair perm[row]], 16-byte vectors, for the rows this
 // call's FFN computes; with expert parallelism the other rows of zero_out
-// (computed by other ranks) are set to zero instead.
+// (computed by other ranks) are set to zero instead.  Before that (packed
+// weights), the gate/up kernel's first weights are brought into L2 as soon
+// as the selected set is published.
 __global__ void __launch_bounds__(256) gather_kernel(const uint16_t *__restrict__ x,
                                                      const int32_t *__restrict__ perm,
                                                      const Meta *__restrict__ meta,
                                                      uint16_t *__restrict__ xp,
                                                      float *__restrict__ zero_out, int B, int d,
-                                                     int k) {
+                                                     int k, GatherPf pf) {
+  __shared__ int32_t s_sel[kMaxN];
+  __shared__ int s_n;
+  if (pf.pk != nullptr && static_cast<int>(blockIdx.x) < kGatherWarmBlocks) warm_gate_up(pf, s_sel, &s_n);
   pdl_wait();
   pdl_trigger();
   const int row = blockIdx.x;
@@ -1470,9 +1569,9 @@ cudaError_t launch_router_logits(const uint16_t *x, const float *Wg, float *h, i
 
 cudaError_t launch_gather(const uint16_t *x, const int32_t *perm, const Meta *meta,
                           uint16_t *xp, float *zero_out, int max_rows, int B, int d, int k,
-                          cudaStream_t s) {
+                          const GatherPf &pf, cudaStream_t s) {
   return launch_pdl(gather_kernel, dim3(max_rows), dim3(256), 0, s, x, perm, meta, xp, zero_out, B,
-                    d, k);
+                    d, k, pf);
 }
 
 cudaError_t launch_combine(const float *out, const int32_t *pos, const float *w,

@@ -103,7 +103,7 @@ __global__ void __launch_bounds__(kRsThreads, 1)
   }
   pdl_wait();
   pdl_trigger();
-  if (cta == 0 && threadIdx.x < 3) done[threadIdx.x] = 0;
+  if (cta == 0 && threadIdx.x < 4) done[threadIdx.x] = 0;
   if (warp == 0) {
     const uint64_t pol_x = policy_evict_last();  // every expert block reads these rows
     for (int i = lane; i < nt * kRsSub; i += 32) {

@@ -106,6 +106,7 @@ __global__ void __launch_bounds__(kThreads, 1) router_tc_kernel(const __grid_con
       p.done[0] = 0;
       p.done[1] = 0;
       p.done[2] = 0;
+      p.done[3] = 0;
     }
     for (int s = 0; s < kMaxStages; ++s) {
       mbar_init(full_bar(s), 1);

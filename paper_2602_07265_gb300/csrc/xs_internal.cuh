@@ -52,6 +52,8 @@ constexpr int kChunk = 32;                   // tokens per selection CTA (= the 
 constexpr int kScatterMaxN = 256;            // parallel stable scatter up to this many experts
 constexpr int kFuseChunks = 2;               // up to this many chunks the selection CTA also refines
 constexpr int kMaxShared = 8;                // shared experts
+constexpr int kGatherPrefetchBytes = 256 * 1024;  // L2 warm-up per gate/up CTA (packed weights)
+constexpr int kGatherWarmBlocks = 32;              // gather blocks that issue the warm-up
 
 // One FFN work tile: up to kTileTok consecutive rows of the permuted pair
 // list, all routed to `expert`.  Experts N .. N + n_shared - 1 are the shared
@@ -121,7 +123,8 @@ struct RouteArgs {
   int32_t *perm_out;
   float *chunk_col;      // [C][N] column-sum tree of each 32-token chunk
   uint8_t *chunk_marks;  // [C][2][N] each chunk's warm-up / base marks and union marks
-  int32_t *done;         // [3] arrival counters (selection, refinement, union), zero at entry
+  int32_t *done;         // [4] arrival counters (selection, refinement, union), zero at
+                         // entry, and the selected-set flag (done[3])
   int32_t *zero_words;   // nullable: region cleared for the FFN kernels
   int zero_count;
   void *const *events;   // nullable: events[0] is recorded between the two kernels
@@ -159,9 +162,20 @@ cudaError_t launch_combine(const float *out, const int32_t *pos, const float *w,
 // Gathers the token rows of this call's FFN rows into xp; with expert
 // parallelism (zero_out != nullptr) it zeroes the rows of zero_out that
 // another rank computes.
+// What the gather kernel needs to warm L2 with the gate/up kernel's first
+// weights (packed weights only; pk == nullptr: no warm-up).
+struct GatherPf {
+  const int32_t *ready;   // done[3]: set by the selection kernel once the mask is written
+  const uint8_t *mask;    // [N] selected set
+  const uint8_t *pk;      // packed gate/up weights
+  int N, MT, KI;          // experts; the gate/up kernel's row blocks and K steps per unit
+  int stage_bytes;        // packed bytes per step (gate and up tiles)
+  int grid;               // the gate/up kernel's grid
+  int pf_bytes;           // bytes per gate/up CTA to prefetch
+};
 cudaError_t launch_gather(const uint16_t *x, const int32_t *perm, const Meta *meta,
                           uint16_t *xp, float *zero_out, int max_rows, int B, int d, int k,
-                          cudaStream_t s);
+                          const GatherPf &pf, cudaStream_t s);
 
 struct FfnArgs {
   const uint16_t *W_gate, *W_up, *W_down;
