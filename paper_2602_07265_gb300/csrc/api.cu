@@ -327,7 +327,9 @@ int xs::forward_impl(const FwdCall &c, FwdStep step) {
     pf.KI = d / 64;
     pf.stage_bytes = 2 * 128 * 64 * 2;
     pf.grid = sms;
-    pf.pf_bytes = kGatherPrefetchBytes;
+    // A refinement kernel of its own (more than kFuseChunks chunks) leaves
+    // a longer window before the gate/up kernel: twice the warm-up.
+    pf.pf_bytes = (B + kChunk - 1) / kChunk > kFuseChunks ? 2 * kGatherPrefetchBytes : kGatherPrefetchBytes;
   }
   if (launch_gather(c.x, a.perm, a.meta, const_cast<uint16_t *>(f.xp), ep ? f.out : nullptr,
                     pl.max_rows, B, d, k, pf, s) != cudaSuccess ||
