@@ -46,6 +46,7 @@ METRIC = "MoE-layer tokens/s and expert-weight HBM GB/s (% roofline); experts ac
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 N_ROTATE = 4   # distinct input batches cycled through the timed steps
+N_SINGLE = 20  # single steps timed one by one for the latency figure
 L2_BYTES = 129e6
 
 
@@ -392,6 +393,18 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
         torch.cuda.synchronize()
     ms_total = reduce_max(ms_local, world, dev)
 
+    # The latency of one layer call: 20 single steps, each between its own
+    # events with the device idle before it (no overlap with a previous
+    # step), median.
+    single_ms = []
+    for i in range(N_SINGLE):
+        a_, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a_.record(stream)
+        step(i)
+        b_.record(stream)
+        torch.cuda.synchronize()
+        single_ms.append(a_.elapsed_time(b_))
+
     st = stats.cpu().numpy()
     if np.any(st[:, 5] != 0):
         raise RuntimeError(f"device status {st[:, 5].max()} (a bounded wait ran out)")
@@ -498,6 +511,8 @@ def run_gpu(args, w: W.Workload, rank: int, world: int, local: int) -> dict:
             "peak_source": peaks["source"],
         },
         "stages_ms": {k: round(v, 5) for k, v in mean_ms.items()},
+        "single_step_ms": {"median": float(np.median(single_ms)), "of": N_SINGLE,
+                           "method": "events around each step, device idle before it"},
         "roofline": {
             "kernel": dominant,
             "bound": "hbm",
