@@ -136,6 +136,12 @@ def test_plain_topk_and_batch_on_workloads(X, name):
     (120, 128, 8, 0, W.MODE_HIER, dict(k0=1, m_r=4, tokens_per_request=8), True),  # 8 | 32
     (144, 64, 4, 5, W.MODE_HIER, dict(k0=2, m_r=2, tokens_per_request=48), False),  # 48 > 32
     (65, 256, 8, 24, W.MODE_BATCH, dict(k0=1), False),                          # 3 chunks, ragged
+    # chunk counts around the refinement kernel (3 to 9 chunks)
+    (257, 256, 8, 24, W.MODE_BATCH, dict(k0=1), False),                         # 9 chunks, ragged
+    (200, 128, 8, 0, W.MODE_THRESH, dict(k0=1, tau=0.6), False),                # 7 chunks, THRESH
+    (160, 64, 8, 0, W.MODE_TOPK, {}, True),                                     # 5 chunks, top-k
+    (100, 64, 8, 3, W.MODE_BATCH, dict(k0=0), False),                           # 4 chunks, |S| < k
+    (96, 64, 8, 0, W.MODE_BATCH, dict(k0=0), False),                            # 3 chunks, S empty
     (64, 256, 8, 0, W.MODE_GROUP, dict(k0=1, n_groups=8, m_g=5), False),        # 2 chunks (fused)
     (256, 256, 8, 0, W.MODE_GROUP, dict(k0=0, n_groups=1, m_g=24), False),     # G = 1 is BATCH
     (256, 256, 8, 0, W.MODE_GROUP, dict(k0=1, n_groups=256, m_g=1), False),    # singleton groups
