@@ -46,7 +46,6 @@ constexpr int kThreads = 192;
 constexpr int kEpiThreads = 128;
 constexpr int kTileBytes = kBM * kBK * 2;     // 16 KB
 constexpr uint64_t kWaitNs = 1000000000ull;   // 1 s per wait
-constexpr int kMinItersPerCta = 8;
 
 template <bool kGateUp>
 struct Cfg {
@@ -154,8 +153,7 @@ __global__ void __launch_bounds__(kThreads, 1) ffn_tc_kernel(const __grid_consta
   Range rg;
   rg.KI = KI;
   rg.I = static_cast<long long>(n_tiles) * MT * KI;
-  const long long want = (rg.I + kMinItersPerCta - 1) / kMinItersPerCta;
-  rg.G = static_cast<int>(want < p.grid ? want : p.grid);
+  rg.G = ffn_ctas(static_cast<long long>(n_tiles) * MT, KI, p.grid);
   if (rg.I == 0 || static_cast<int>(blockIdx.x) >= rg.G) {
     pdl_wait();
     pdl_trigger();

@@ -1349,11 +1349,11 @@ __global__ void __launch_bounds__(kRtWarps * 32) router_logits_kernel(
 
 // L2 warm-up for the gate/up kernel (packed weights).  Its stream-K split
 // and segment order are those of ffn_tc.cu, predicted from the selected set
-// (one tile per selected expert, in expert order): CTA c of G takes steps
-// [I c / G, I (c + 1) / G) of I = |S| x MT x KI and does first the steps of
-// its last unit (if that unit continues in CTA c + 1), then those of its
-// first unit (if it began in CTA c - 1), then its whole units.  The first
-// pf_bytes of that order are prefetched into L2, by the first
+// (one tile per selected expert, in expert order): CTA c of G = ffn_ctas()
+// takes steps [I c / G, I (c + 1) / G) of I = |S| x MT x KI and does first
+// the steps of its last unit (if that unit continues in CTA c + 1), then
+// those of its first unit (if it began in CTA c - 1), then its whole units.
+// The first pf_bytes of that order are prefetched into L2, by the first
 // kGatherWarmBlocks blocks (a few gate/up CTAs' ranges each: fewer blocks
 // waiting on the flag and a less bursty stream of prefetches measured
 // faster than one block per gate/up CTA).  A wrong prediction (an expert of
@@ -1392,8 +1392,7 @@ __device__ void warm_gate_up(const GatherPf &g, int32_t *s_sel, int *s_n) {
   const int nS = *s_n;
   if (nS <= 0) return;
   const long long KI = g.KI, I = static_cast<long long>(nS) * g.MT * KI;
-  const long long want = (I + 7) / 8;  // the FFN kernel's minimum of 8 steps per CTA
-  const int G = static_cast<int>(want < g.grid ? want : g.grid);
+  const int G = ffn_ctas(static_cast<long long>(nS) * g.MT, g.KI, g.grid);  // gate/up CTAs
   const int n_steps = g.pf_bytes / g.stage_bytes;
   const int nb = gridDim.x < kGatherWarmBlocks ? static_cast<int>(gridDim.x) : kGatherWarmBlocks;
   for (int c = blockIdx.x; c < G; c += nb) {

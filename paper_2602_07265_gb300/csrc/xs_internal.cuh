@@ -55,6 +55,26 @@ constexpr int kMaxShared = 8;                // shared experts
 constexpr int kGatherPrefetchBytes = 256 * 1024;  // L2 warm-up per gate/up CTA (packed weights)
 constexpr int kGatherWarmBlocks = 32;              // gather blocks that issue the warm-up
 
+// CTAs an FFN kernel splits its U units (a token tile x 128 weight rows, KI
+// K steps each) over, at most `grid`.  Stream-K gives CTA c the steps
+// [I c / G, I (c + 1) / G) of I = U KI, at least kFfnMinSteps each; a unit
+// cut between CTAs is finished from partial sums.  When q = ceil(U / grid)
+// is 1 or 2, divides U, and G = U / q CTAs still cover 80 % of the SMs, G is
+// that: every range then ends on a unit boundary and no unit is cut (no
+// partial sums, no reductions), which measured OLMoE B = 8 at 58.7 -> 52.5 us
+// on GB300.  With more units per CTA or more idle SMs the cuts cost less
+// than the longer per-CTA stream (DeepSeek-R1 B = 8 on 81 % of the SMs, five
+// units each: 398 -> 409 us).  The gather kernel's L2 warm-up predicts the
+// gate/up split with the same function.
+constexpr int kFfnMinSteps = 8;
+__host__ __device__ inline int ffn_ctas(long long U, int KI, int grid) {
+  const long long I = U * KI, want = (I + kFfnMinSteps - 1) / kFfnMinSteps;
+  const long long q = (U + grid - 1) / grid;
+  if (U > 0 && q <= 2 && U % q == 0 && (U / q) * 5 >= static_cast<long long>(grid) * 4)
+    return static_cast<int>(U / q);
+  return static_cast<int>(want < grid ? want : grid);
+}
+
 // One FFN work tile: up to kTileTok consecutive rows of the permuted pair
 // list, all routed to `expert`.  Experts N .. N + n_shared - 1 are the shared
 // experts; their rows follow the routed pairs: row n_pairs + j * B + t is
